@@ -1,0 +1,221 @@
+/*
+ * taps.h - C ABI of the TAPS per-round hot path on one GB300 (sm_103a).
+ *
+ * TAPS (Target-Aware Prefix tree Selection, diffusion-drafted speculative
+ * decoding) runs one decoding round in six steps; each has one entry point:
+ *
+ *   taps_topk_marginals    Sec. 4.1 stage 1 + Sec. 4.2 features
+ *   taps_score_reach       Sec. 4.2, Eq. 1, Algorithm 1 (scorer + sibling softmax)
+ *   taps_select_subtree    Sec. 4.2-4.3, Eq. 2, Eq. 3, Algorithm 1 (selection)
+ *   taps_build_tree_mask   Sec. 4.1 stage 3 / Sec. 4.3 (tree attention needs
+ *                          a connected subtree rooted at the current position)
+ *   taps_tree_verify_attn  Sec. 4.1 stage 3 (target verifies the subtree with
+ *                          tree attention), over a paged bf16 KV cache
+ *   taps_accept            Sec. 4.1 and Limitations (greedy, temperature 0,
+ *                          lossless acceptance of the longest matching path)
+ *
+ * Conventions shared by every call:
+ *  - Array arguments are DEVICE pointers owned by the caller. The library never
+ *    allocates, frees or synchronises; every call is asynchronous on `stream`
+ *    (a cudaStream_t passed as void*, NULL = legacy default stream).
+ *  - Parameter structs are HOST pointers, read before the call returns.
+ *  - Arrays are dense, row-major, in the shapes given; B = requests,
+ *    L = drafted positions (tree depth), V = vocabulary, K = top-K per
+ *    position, N = n_max node budget (root included).
+ *  - Return value is a taps_status. Host-side argument checks run before any
+ *    launch; on any error nothing is launched and outputs are untouched.
+ *    TAPS_ERR_CUDA reports a launch failure (cudaGetLastError).
+ *  - Device-detected faults (an out-of-range page id) never trap: the kernel
+ *    skips the bad access and ORs a TAPS_DEVFAULT_* bit into the caller's
+ *    `status` word (nullable), which the caller reads after synchronising.
+ *  - Workspaces are caller-allocated device buffers of at least the size the
+ *    matching *_workspace_bytes() query returns, 256-byte aligned and
+ *    ZERO-FILLED before their first use; every call leaves the counters it
+ *    uses back at zero. Calls that share a workspace must not overlap.
+ */
+#ifndef TAPS_H_
+#define TAPS_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum taps_status {
+  TAPS_OK = 0,
+  TAPS_ERR_INVALID_ARG = 1,   /* null pointer, negative size, inconsistent shape */
+  TAPS_ERR_UNSUPPORTED = 2,   /* outside the supported limits listed per call   */
+  TAPS_ERR_WORKSPACE = 3,     /* workspace missing, too small or misaligned     */
+  TAPS_ERR_CUDA = 4,          /* a kernel launch failed                         */
+  TAPS_ERR_DEVICE = 5         /* reserved for device-detected faults            */
+} taps_status;
+
+enum { TAPS_F32 = 0, TAPS_BF16 = 1 };
+enum { TAPS_SCORER_MARGINAL = 0, TAPS_SCORER_MLP = 1 };
+enum { TAPS_DEVFAULT_PAGE = 1 };
+
+/* Limits (TAPS_ERR_UNSUPPORTED beyond them). */
+#define TAPS_MAX_K 32
+#define TAPS_MAX_L 31
+#define TAPS_MAX_V 262143      /* token ids must fit in 18 bits */
+#define TAPS_MAX_NODES 512
+#define TAPS_MAX_EMB 32
+#define TAPS_MAX_HIDDEN 64
+
+const char* taps_status_string(int status);
+int taps_version(void);
+
+/* ------------------------------------------------------------------------
+ * taps_topk_marginals - Sec. 4.1 stage 1 (the top-K tokens of every drafted
+ * position form the candidate tree) and Sec. 4.2 (the scorer reads the child
+ * log-probability and the positional entropy).
+ *
+ * logits     [B, L, V] of dtype TAPS_F32 or TAPS_BF16; row (b, d) starts at
+ *            element (b * L + d) * row_stride (row_stride >= V).
+ * topk_ids   [B, L, K] int32, out: the K largest logits of each row, ordered
+ *            by logit descending, then token id ascending.
+ * topk_logp  [B, L, K] f32, out: logit - lse (full-vocabulary log-probability).
+ * lse        [B, L] f32, out: log sum_v exp(logit_v).
+ * entropy    [B, L] f32, out: -sum_v p_v log p_v in nats, full vocabulary.
+ * ws         workspace of taps_topk_marginals_workspace_bytes(B, L, V, K).
+ * Limits: 1 <= K <= min(32, V), 1 <= V <= 262143. Logits must be finite.
+ * ---------------------------------------------------------------------- */
+size_t taps_topk_marginals_workspace_bytes(int B, int L, int V, int K);
+int taps_topk_marginals(const void* logits, int dtype, int64_t row_stride,
+                        int B, int L, int V, int K,
+                        int32_t* topk_ids, float* topk_logp, float* lse, float* entropy,
+                        void* ws, size_t ws_bytes, void* stream);
+
+/* ------------------------------------------------------------------------
+ * taps_score_reach - Sec. 4.2, Eq. 1 and Algorithm 1: for every parent of
+ * the candidate trie, q_cond(parent -> child) = softmax over the K siblings
+ * of the scorer logit of each edge.
+ *
+ * The candidate trie: every node at depth d has the same K children, the
+ * top-K tokens of position d; the root (depth 0) carries root_tok[b].
+ * q_cond[b, d, i, j] (f32 [B, L, K, K], out) is the conditional acceptance
+ * of child slot j of position d given that parent slot i of position d-1 was
+ * reached; for d == 0 the parent is the root, row i = 0, and rows i >= 1 are
+ * written as 0.
+ *
+ * Scorer (params->kind):
+ *  TAPS_SCORER_MARGINAL  logit = topk_logp[b, d, j] (the paper's ablation that
+ *                        ranks by the drafter's marginal confidence, Sec. 5.3).
+ *  TAPS_SCORER_MLP       logit = w_lp * logp + w2 . relu(W1 f + b1) with
+ *                        f = [E_tok[parent], E_tok[child], E_dep[d+1], logp,
+ *                        entropy[b, d]] (Sec. 4.2 feature list). weights is a
+ *                        device f32 buffer: tok_emb[vocab][E], dep_emb[max_depth][E],
+ *                        W1[H][3E+2], b1[H], w2[H], w_lp[1], packed in that
+ *                        order. Token ids must be < vocab; max_depth > L.
+ * Limits: K <= 32, L <= 31, E <= 32, H <= 64.
+ * ---------------------------------------------------------------------- */
+typedef struct taps_scorer_params {
+  int kind;
+  int emb_dim;     /* E */
+  int hidden;      /* H */
+  int vocab;       /* rows of tok_emb */
+  int max_depth;   /* rows of dep_emb */
+  const float* weights;
+} taps_scorer_params;
+
+int taps_score_reach(const int32_t* root_tok, const int32_t* topk_ids, const float* topk_logp,
+                     const float* entropy, int B, int L, int K,
+                     const taps_scorer_params* params, float* q_cond, void* stream);
+
+/* ------------------------------------------------------------------------
+ * taps_select_subtree - Eq. 2 (reach = product of q_cond along the path),
+ * Eq. 3 (utility = reach / (lambda1 + lambda2 * depth)) and Algorithm 1:
+ * starting from S = {root}, repeatedly add the unselected node of largest
+ * utility while |S| < n_max and that utility > tau.
+ *
+ * Arithmetic: reach and utility are f32 with IEEE round-to-nearest multiply
+ * and divide, accumulated root to leaf; den(d) = lambda1 + lambda2 * d.
+ * Ties: utility descending, then depth ascending, then token id ascending,
+ * then the parent's position in the selection order ascending.
+ * Outputs ([B, n_max] unless noted), nodes listed in the order the greedy
+ * loop adds them (root = node 0, parent[i] < i); entries at i >= n_nodes[b]
+ * are -1 (int) or 0 (float):
+ *   n_nodes [B], parent, depth, token (root = root_tok[b]), slot (top-K slot
+ *   of the node's position, root = -1), pos_id (= ctx_len[b] + depth),
+ *   reach, utility.
+ * Requires q_cond entries in [0, 1] (as taps_score_reach produces), lambda1 > 0,
+ * lambda2 >= 0, tau >= 0, 1 <= n_max <= 512, K <= 32, L <= 31.
+ * ---------------------------------------------------------------------- */
+typedef struct taps_select_params {
+  float lambda1;
+  float lambda2;
+  float tau;
+  int n_max;
+} taps_select_params;
+
+int taps_select_subtree(const float* q_cond, const int32_t* topk_ids, const int32_t* root_tok,
+                        const int32_t* ctx_len, int B, int L, int K,
+                        const taps_select_params* params,
+                        int32_t* n_nodes, int32_t* parent, int32_t* depth, int32_t* token,
+                        int32_t* slot, int32_t* pos_id, float* reach, float* utility,
+                        void* stream);
+
+/* ------------------------------------------------------------------------
+ * taps_build_tree_mask - the ancestor-or-self relation that tree attention
+ * needs (Sec. 4.1 stage 3, Sec. 4.3).
+ *
+ * mask [B, n_max, ceil(n_max / 32)] uint32, out: bit (j % 32) of word j / 32
+ * of row i is 1 iff i, j < n_nodes[b] and j is i or an ancestor of i.
+ * parent [B, n_max] as written by taps_select_subtree.
+ * ---------------------------------------------------------------------- */
+int taps_build_tree_mask(const int32_t* parent, const int32_t* n_nodes, int B, int n_max,
+                         uint32_t* mask, void* stream);
+
+/* ------------------------------------------------------------------------
+ * taps_tree_verify_attn - tree attention of the selected nodes against the
+ * target's KV cache (Sec. 4.1 stage 3): for node i and query head h (KV head
+ * h / (Hq / Hkv)),
+ *   out = softmax(scale * q K^T over visible positions) V,
+ * where the visible positions are the whole context [0, ctx_len[b]) and the
+ * tree positions ctx_len[b] + j with bit j set in mask row i.
+ *
+ * q        [B, n_max, Hq, D] bf16 (post-RoPE queries of the tree nodes).
+ * k_cache, v_cache [num_pages, Hkv, page_size, D] bf16. Logical position t
+ *          of request b lives in page block_table[b * max_pages + t / page_size],
+ *          row t % page_size. Tree node j's K/V must already sit at logical
+ *          position ctx_len[b] + j, so pages must cover ctx_len[b] + n_nodes[b].
+ * out      [B, n_max, Hq, D] bf16, out; rows i >= n_nodes[b] are written as 0.
+ * lse_out  [B, n_max, Hq] f32, out, nullable: natural-log softmax denominator.
+ * max_ctx  host upper bound of ctx_len[b] (sizes the split of the context).
+ * ws       workspace of taps_tree_verify_attn_workspace_bytes(...).
+ * status   device int32, nullable: TAPS_DEVFAULT_PAGE is ORed in when a page
+ *          id is outside [0, num_pages); that page is then skipped.
+ * Limits: D in {64, 128}, page_size == 16, Hq % Hkv == 0, Hq / Hkv <= 8,
+ *         n_max <= 512.
+ * ---------------------------------------------------------------------- */
+size_t taps_tree_verify_attn_workspace_bytes(int B, int n_max, int Hq, int Hkv, int D,
+                                             int max_ctx);
+int taps_tree_verify_attn(const void* q, const void* k_cache, const void* v_cache,
+                          int64_t num_pages, const int32_t* block_table, int max_pages,
+                          const int32_t* ctx_len, const int32_t* n_nodes, const uint32_t* mask,
+                          int B, int n_max, int Hq, int Hkv, int D, int page_size, float scale,
+                          int max_ctx, void* out, float* lse_out,
+                          void* ws, size_t ws_bytes, int32_t* status, void* stream);
+
+/* ------------------------------------------------------------------------
+ * taps_accept - lossless greedy acceptance (Sec. 4.1, Limitations): from the
+ * root, step into the child whose token equals the target's greedy token at
+ * the current node, until no child matches.
+ *
+ * target_tok [B, n_max] int32: the target model's greedy next token after
+ *          the prefix ending at node i.
+ * accept_len [B] out: accepted draft tokens (depth of the last accepted node).
+ * accepted_nodes [B, L + 1] out: node indices root .. last, then -1.
+ * bonus_tok [B] out: target_tok at the last accepted node.
+ * ---------------------------------------------------------------------- */
+int taps_accept(const int32_t* parent, const int32_t* token, const int32_t* n_nodes,
+                const int32_t* target_tok, int B, int n_max, int L,
+                int32_t* accept_len, int32_t* accepted_nodes, int32_t* bonus_tok, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* TAPS_H_ */

@@ -294,7 +294,8 @@ def build_tree_mask(parent, n_nodes, n_max):
 # Stage 5: tree-masked verification attention over a paged KV cache
 # ---------------------------------------------------------------------------
 
-def tree_verify_attn(q, k_cache, v_cache, block_table, ctx_len, n_nodes, mask, scale=None):
+def tree_verify_attn(q, k_cache, v_cache, block_table, ctx_len, n_nodes, mask, scale=None,
+                     only=None):
     """Textbook masked softmax attention of every tree node, in float64.
 
     q: [B, N, Hq, D]; k_cache, v_cache: [num_pages, Hkv, P, D]; logical
@@ -302,6 +303,8 @@ def tree_verify_attn(q, k_cache, v_cache, block_table, ctx_len, n_nodes, mask, s
     attends to positions [0, ctx_len) and to ctx_len + j for every j set in
     mask[b, i]. Returns out [B, N, Hq, D] and lse [B, N, Hq] (natural log of
     the softmax denominator of the scaled scores); rows i >= n_nodes are 0.
+    ``only``: optional set of (b, i, h) triples; other outputs are left 0 (a
+    way to sample single outputs of a large case, same arithmetic).
     """
     q = np.asarray(q, np.float64)
     B, N, Hq, D = q.shape
@@ -312,6 +315,8 @@ def tree_verify_attn(q, k_cache, v_cache, block_table, ctx_len, n_nodes, mask, s
     lse = np.zeros((B, N, Hq), np.float64)
     for b in range(B):
         C, n = int(ctx_len[b]), int(n_nodes[b])
+        if only is not None and not any(o[0] == b for o in only):
+            continue
         T = C + n
         t = np.arange(T)
         pages = block_table[b, t // P]
@@ -324,6 +329,8 @@ def tree_verify_attn(q, k_cache, v_cache, block_table, ctx_len, n_nodes, mask, s
                 if (int(mask[b, i, j // 32]) >> (j % 32)) & 1:
                     visible[C + j] = True
             for h in range(Hq):
+                if only is not None and (b, i, h) not in only:
+                    continue
                 kv = h // group
                 s = scale * (Kb[visible, kv, :] @ q[b, i, h])
                 m = s.max()

@@ -1,0 +1,381 @@
+// Stage 1 of a TAPS round (Sec. 4.1 stage 1, Sec. 4.2 scorer features):
+// per-position full-vocabulary softmax statistics and top-K candidates.
+//
+// One pass over the logits. Each row (request b, position d) is split into
+// `chunks` contiguous slices, one CTA each, so that a batch-1 round still
+// spreads over every SM. A CTA reads its slice with 16-byte vector loads,
+// keeps per-thread running statistics (max, sum of exponentials, sum of
+// exponential-weighted offsets for the entropy) and a per-thread sorted top-K
+// list of 64-bit keys (ordered logit << 32 | ~token id), merges them with warp
+// redux operations, and writes one partial record. The last CTA of a row (an
+// atomic ticket, reset after use) merges the partials and writes the row's
+// outputs. No CTA waits on another.
+#include <algorithm>
+
+#include "common.cuh"
+
+namespace taps {
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kWarps = kThreads / 32;
+constexpr int kMaxChunks = 64;
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.6931471805599453f;
+
+struct Plan {
+  int rows, chunks, kp;
+};
+
+int round_kp(int K) {
+  int kp = 1;
+  while (kp < K) kp <<= 1;
+  return kp;
+}
+
+Plan make_plan(int B, int L, int V, int K) {
+  Plan p;
+  p.rows = B * L;
+  p.kp = round_kp(K);
+  int want = (4 * kTargetSms + p.rows - 1) / p.rows;
+  int maxc = std::max(1, V / 2048);
+  p.chunks = std::max(1, std::min(want, std::min(maxc, kMaxChunks)));
+  return p;
+}
+
+struct WsLayout {
+  size_t stats, keys, tickets, total;
+};
+
+WsLayout ws_layout(const Plan& p) {
+  WsLayout w;
+  size_t o = 0;
+  w.stats = o;
+  o = align_up(o + sizeof(float4) * p.rows * p.chunks, 256);
+  w.keys = o;
+  o = align_up(o + sizeof(uint64_t) * p.rows * p.chunks * p.kp, 256);
+  w.tickets = o;
+  o = align_up(o + sizeof(unsigned) * p.rows, 256);
+  w.total = o;
+  return w;
+}
+
+// Running softmax statistics in log2 units: m2 = max x*log2(e),
+// z = sum 2^(x2 - m2), t2 = sum 2^(x2 - m2) * (x2 - m2).
+struct Stats {
+  float m2, z, t2;
+};
+
+__device__ __forceinline__ void stats_raise(Stats& s, float m2_new) {
+  if (m2_new > s.m2) {
+    if (s.z > 0.f) {
+      float dm = s.m2 - m2_new;
+      float sc = exp2f(dm);
+      s.t2 = sc * fmaf(s.z, dm, s.t2);
+      s.z *= sc;
+    }
+    s.m2 = m2_new;
+  }
+}
+
+__device__ __forceinline__ void stats_add(Stats& s, float x2) {
+  if (x2 > -INFINITY) {
+    float dx = x2 - s.m2;
+    float e = exp2f(dx);
+    s.z += e;
+    s.t2 = fmaf(e, dx, s.t2);
+  }
+}
+
+__device__ __forceinline__ Stats stats_merge(Stats a, Stats b) {
+  float m = fmaxf(a.m2, b.m2);
+  Stats r{m, 0.f, 0.f};
+  if (a.z > 0.f) {
+    float d = a.m2 - m;
+    float s = exp2f(d);
+    r.z += s * a.z;
+    r.t2 += s * fmaf(a.z, d, a.t2);
+  }
+  if (b.z > 0.f) {
+    float d = b.m2 - m;
+    float s = exp2f(d);
+    r.z += s * b.z;
+    r.t2 += s * fmaf(b.z, d, b.t2);
+  }
+  return r;
+}
+
+template <int KP>
+__device__ __forceinline__ void list_insert(uint64_t (&lst)[KP], uint64_t key) {
+  if (key <= lst[KP - 1]) return;
+#pragma unroll
+  for (int i = 0; i < KP; ++i) {
+    if (key > lst[i]) {
+      uint64_t t = lst[i];
+      lst[i] = key;
+      key = t;
+    }
+  }
+}
+
+__device__ __forceinline__ uint64_t make_key(float x, uint32_t id) {
+  return (static_cast<uint64_t>(f32_to_ordered(x)) << 32) | static_cast<uint32_t>(~id);
+}
+
+template <typename T>
+__device__ __forceinline__ float to_f32(T v);
+template <>
+__device__ __forceinline__ float to_f32<float>(float v) { return v; }
+template <>
+__device__ __forceinline__ float to_f32<__nv_bfloat16>(__nv_bfloat16 v) {
+  return __bfloat162float(v);
+}
+
+template <int KP, typename T>
+__device__ __forceinline__ void consume(float x, uint32_t id, Stats& st, uint64_t (&lst)[KP]) {
+  stats_add(st, x * kLog2e);
+  list_insert<KP>(lst, make_key(x, id));
+}
+
+// Merge KP rounds over `count` unsorted keys in shared memory (one warp).
+template <int KP>
+__device__ void warp_select_smem(uint64_t* cand, int count, uint64_t* out, int lane) {
+  for (int r = 0; r < KP; ++r) {
+    uint64_t mine = 0;
+    int mi = -1;
+    for (int i = lane; i < count; i += 32) {
+      uint64_t v = cand[i];
+      if (v > mine) {
+        mine = v;
+        mi = i;
+      }
+    }
+    uint64_t best = warp_max_u64(mine);
+    if (best != 0 && mine == best) cand[mi] = 0;
+    if (lane == 0) out[r] = best;
+    __syncwarp();
+  }
+}
+
+__device__ __forceinline__ Stats warp_stats(Stats s) {
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    Stats o;
+    o.m2 = __shfl_xor_sync(kFullMask, s.m2, off);
+    o.z = __shfl_xor_sync(kFullMask, s.z, off);
+    o.t2 = __shfl_xor_sync(kFullMask, s.t2, off);
+    s = stats_merge(s, o);
+  }
+  return s;
+}
+
+template <int KP>
+__device__ void write_row(int row, int K, const uint64_t* top, Stats st, int lane,
+                          int32_t* ids, float* logp, float* lse, float* ent) {
+  float xmax = ordered_to_f32(static_cast<uint32_t>(top[0] >> 32));
+  float lz = logf(st.z);
+  float l = xmax + lz;
+  if (lane == 0) {
+    lse[row] = l;
+    ent[row] = lz - (st.t2 * kLn2) / st.z;
+  }
+  for (int k = lane; k < K; k += 32) {
+    uint64_t key = top[k];
+    ids[static_cast<int64_t>(row) * K + k] = static_cast<int32_t>(~static_cast<uint32_t>(key));
+    logp[static_cast<int64_t>(row) * K + k] =
+        ordered_to_f32(static_cast<uint32_t>(key >> 32)) - l;
+  }
+}
+
+template <int KP, typename T>
+__global__ void __launch_bounds__(kThreads)
+topk_marginals_kernel(const T* __restrict__ logits, int64_t row_stride, int V, int K, int chunks,
+                      int vec_ok, int32_t* __restrict__ ids, float* __restrict__ logp,
+                      float* __restrict__ lse, float* __restrict__ ent, float4* ws_stats,
+                      uint64_t* ws_keys, unsigned* tickets) {
+  constexpr int VE = 16 / sizeof(T);
+  __shared__ uint64_t s_cand[kMaxChunks * 32];
+  __shared__ uint64_t s_top[32];
+  __shared__ Stats s_wstats[kWarps];
+  __shared__ int s_last;
+
+  const int row = blockIdx.y;
+  const int chunk = blockIdx.x;
+  const int tid = threadIdx.x;
+  const int lane = tid & 31;
+  const int warp = tid >> 5;
+  const T* x = logits + static_cast<int64_t>(row) * row_stride;
+
+  Stats st{-INFINITY, 0.f, 0.f};
+  uint64_t lst[KP];
+#pragma unroll
+  for (int i = 0; i < KP; ++i) lst[i] = 0;
+
+  if (vec_ok) {
+    const int nvec = V / VE;
+    const int per = (nvec + chunks - 1) / chunks;
+    const int v0 = chunk * per;
+    const int v1 = min(nvec, v0 + per);
+    const uint4* xv = reinterpret_cast<const uint4*>(x);
+    constexpr int U = 4;
+    for (int base = v0 + tid; base < v1; base += U * kThreads) {
+      uint4 buf[U];
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        int v = base + u * kThreads;
+        if (v < v1) buf[u] = __ldcs(xv + v);
+      }
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        int v = base + u * kThreads;
+        if (v < v1) {
+          const T* e = reinterpret_cast<const T*>(&buf[u]);
+          float vals[VE];
+          float vmax = -INFINITY;
+#pragma unroll
+          for (int i = 0; i < VE; ++i) {
+            vals[i] = to_f32<T>(e[i]);
+            vmax = fmaxf(vmax, vals[i]);
+          }
+          stats_raise(st, vmax * kLog2e);
+#pragma unroll
+          for (int i = 0; i < VE; ++i)
+            consume<KP, T>(vals[i], static_cast<uint32_t>(v * VE + i), st, lst);
+        }
+      }
+    }
+    // tail elements past the last full vector go to the last chunk
+    if (chunk == chunks - 1) {
+      for (int i = nvec * VE + tid; i < V; i += kThreads) {
+        float xv1 = to_f32<T>(x[i]);
+        stats_raise(st, xv1 * kLog2e);
+        consume<KP, T>(xv1, static_cast<uint32_t>(i), st, lst);
+      }
+    }
+  } else {
+    const int per = (V + chunks - 1) / chunks;
+    const int e0 = chunk * per;
+    const int e1 = min(V, e0 + per);
+    for (int i = e0 + tid; i < e1; i += kThreads) {
+      float xv1 = to_f32<T>(x[i]);
+      stats_raise(st, xv1 * kLog2e);
+      consume<KP, T>(xv1, static_cast<uint32_t>(i), st, lst);
+    }
+  }
+
+  // ---- warp merge: KP rounds of a 64-bit warp maximum over list heads
+  for (int r = 0; r < KP; ++r) {
+    uint64_t best = warp_max_u64(lst[0]);
+    if (lane == 0) s_cand[warp * KP + r] = best;
+    if (best != 0 && lst[0] == best) {
+#pragma unroll
+      for (int i = 0; i < KP - 1; ++i) lst[i] = lst[i + 1];
+      lst[KP - 1] = 0;
+    }
+  }
+  st = warp_stats(st);
+  if (lane == 0) s_wstats[warp] = st;
+  __syncthreads();
+
+  if (warp == 0) {
+    warp_select_smem<KP>(s_cand, kWarps * KP, s_top, lane);
+    Stats cs = s_wstats[0];
+    for (int w = 1; w < kWarps; ++w) cs = stats_merge(cs, s_wstats[w]);
+    if (chunks == 1) {
+      __syncwarp();
+      write_row<KP>(row, K, s_top, cs, lane, ids, logp, lse, ent);
+    } else {
+      const int64_t rec = static_cast<int64_t>(row) * chunks + chunk;
+      if (lane == 0) ws_stats[rec] = make_float4(cs.m2, cs.z, cs.t2, 0.f);
+      __syncwarp();
+      for (int r = lane; r < KP; r += 32) ws_keys[rec * KP + r] = s_top[r];
+      __threadfence();
+      __syncwarp();
+      if (lane == 0) s_last = (atomicAdd(&tickets[row], 1u) == static_cast<unsigned>(chunks - 1));
+      __syncwarp();
+    }
+  }
+  if (chunks == 1) return;
+  __syncthreads();
+  if (!s_last) return;
+
+  // ---- last CTA of this row: merge every chunk's partial record
+  __threadfence();
+  const int64_t rec0 = static_cast<int64_t>(row) * chunks;
+  for (int i = tid; i < chunks * KP; i += kThreads) s_cand[i] = __ldcg(ws_keys + rec0 * KP + i);
+  __syncthreads();
+  if (warp == 0) {
+    Stats cs{-INFINITY, 0.f, 0.f};
+    for (int c = lane; c < chunks; c += 32) {
+      float4 p = __ldcg(ws_stats + rec0 + c);
+      cs = stats_merge(cs, Stats{p.x, p.y, p.z});
+    }
+    cs = warp_stats(cs);
+    warp_select_smem<KP>(s_cand, chunks * KP, s_top, lane);
+    __syncwarp();
+    write_row<KP>(row, K, s_top, cs, lane, ids, logp, lse, ent);
+    if (lane == 0) tickets[row] = 0u;
+  }
+}
+
+template <int KP, typename T>
+void launch(const void* logits, int64_t row_stride, const Plan& p, int V, int K, int vec_ok,
+            int32_t* ids, float* logp, float* lse, float* ent, char* ws, const WsLayout& w,
+            cudaStream_t s) {
+  dim3 grid(p.chunks, p.rows);
+  float4* st = p.chunks > 1 ? reinterpret_cast<float4*>(ws + w.stats) : nullptr;
+  uint64_t* keys = p.chunks > 1 ? reinterpret_cast<uint64_t*>(ws + w.keys) : nullptr;
+  unsigned* tk = p.chunks > 1 ? reinterpret_cast<unsigned*>(ws + w.tickets) : nullptr;
+  topk_marginals_kernel<KP, T><<<grid, kThreads, 0, s>>>(
+      static_cast<const T*>(logits), row_stride, V, K, p.chunks, vec_ok, ids, logp, lse, ent,
+      st, keys, tk);
+}
+
+template <typename T>
+void dispatch_kp(int kp, const void* logits, int64_t row_stride, const Plan& p, int V, int K,
+                 int vec_ok, int32_t* ids, float* logp, float* lse, float* ent, char* ws,
+                 const WsLayout& w, cudaStream_t s) {
+  switch (kp) {
+    case 1: launch<1, T>(logits, row_stride, p, V, K, vec_ok, ids, logp, lse, ent, ws, w, s); break;
+    case 2: launch<2, T>(logits, row_stride, p, V, K, vec_ok, ids, logp, lse, ent, ws, w, s); break;
+    case 4: launch<4, T>(logits, row_stride, p, V, K, vec_ok, ids, logp, lse, ent, ws, w, s); break;
+    case 8: launch<8, T>(logits, row_stride, p, V, K, vec_ok, ids, logp, lse, ent, ws, w, s); break;
+    case 16: launch<16, T>(logits, row_stride, p, V, K, vec_ok, ids, logp, lse, ent, ws, w, s); break;
+    default: launch<32, T>(logits, row_stride, p, V, K, vec_ok, ids, logp, lse, ent, ws, w, s); break;
+  }
+}
+
+}  // namespace
+}  // namespace taps
+
+using namespace taps;
+
+extern "C" size_t taps_topk_marginals_workspace_bytes(int B, int L, int V, int K) {
+  if (B <= 0 || L <= 0 || V <= 0 || K <= 0 || K > TAPS_MAX_K) return 0;
+  return ws_layout(make_plan(B, L, V, K)).total;
+}
+
+extern "C" int taps_topk_marginals(const void* logits, int dtype, int64_t row_stride, int B,
+                                   int L, int V, int K, int32_t* topk_ids, float* topk_logp,
+                                   float* lse, float* entropy, void* ws, size_t ws_bytes,
+                                   void* stream) {
+  if (!logits || !topk_ids || !topk_logp || !lse || !entropy) return TAPS_ERR_INVALID_ARG;
+  if (B <= 0 || L <= 0 || V <= 0 || K <= 0 || row_stride < V) return TAPS_ERR_INVALID_ARG;
+  if (dtype != TAPS_F32 && dtype != TAPS_BF16) return TAPS_ERR_INVALID_ARG;
+  if (K > TAPS_MAX_K || K > V || V > TAPS_MAX_V) return TAPS_ERR_UNSUPPORTED;
+  if (static_cast<int64_t>(B) * L > 65535) return TAPS_ERR_UNSUPPORTED;
+  Plan p = make_plan(B, L, V, K);
+  WsLayout w = ws_layout(p);
+  if (p.chunks > 1 && (!ws || ws_bytes < w.total || !aligned(ws, 256))) return TAPS_ERR_WORKSPACE;
+  const size_t esz = dtype == TAPS_F32 ? 4 : 2;
+  const int vec_ok = aligned(logits, 16) && (row_stride * esz) % 16 == 0;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  char* wsc = static_cast<char*>(ws);
+  if (dtype == TAPS_F32)
+    dispatch_kp<float>(p.kp, logits, row_stride, p, V, K, vec_ok, topk_ids, topk_logp, lse,
+                       entropy, wsc, w, s);
+  else
+    dispatch_kp<__nv_bfloat16>(p.kp, logits, row_stride, p, V, K, vec_ok, topk_ids, topk_logp,
+                               lse, entropy, wsc, w, s);
+  return launch_status();
+}

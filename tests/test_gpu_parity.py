@@ -1,0 +1,463 @@
+"""Parity of every CUDA stage (through the C ABI) with the CPU oracle.
+
+Tolerances (derived in the design doc):
+* integer results (top-K ids, tree topology, mask, acceptance) bit-exact;
+* lse, entropy: 1e-5 relative; logp = logit - lse: 1e-5 of max(|logp|, |lse|);
+* q_cond (same inputs on both sides): 1e-5 relative, 1e-7 absolute floor;
+* reach and utility from the same q_cond: bit-exact (same f32 IEEE operations);
+* attention outputs (bf16): 2e-2 absolute against the float64 oracle.
+"""
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+
+pytestmark = pytest.mark.gpu
+
+import workloads as W  # noqa: E402
+from oracle import taps_oracle as O  # noqa: E402
+
+ATTN_ATOL = 2e-2
+
+
+@pytest.fixture(scope="module")
+def taps():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import __graft_entry__
+    __graft_entry__.build()
+    import paper_2606_00487_gb300 as t
+    return t
+
+
+DEV = "cuda:0"
+
+
+def dt(a):
+    return torch.from_numpy(np.ascontiguousarray(a)).to(DEV)
+
+
+def bf(a):
+    return dt(np.asarray(a, np.float32)).to(torch.bfloat16)
+
+
+def host(t):
+    return t.cpu().numpy()
+
+
+# ---------------------------------------------------------------------------
+# Stage 1
+# ---------------------------------------------------------------------------
+
+def _check_topk(taps, x, K, dtype=torch.float32, x_dev=None):
+    xd = x_dev if x_dev is not None else dt(x.astype(np.float32)).to(dtype)
+    ids, logp, lse, ent = taps.taps_topk_marginals(xd, K)
+    torch.cuda.synchronize()
+    r_ids, r_logp, r_lse, r_ent = O.topk_marginals(x, K)
+    np.testing.assert_array_equal(host(ids), r_ids)
+    np.testing.assert_allclose(host(lse), r_lse, rtol=1e-5)
+    np.testing.assert_allclose(host(ent), r_ent, rtol=1e-5, atol=1e-6)
+    scale = np.maximum(np.abs(r_logp), np.abs(r_lse)[..., None])
+    assert np.all(np.abs(host(logp) - r_logp) <= 1e-5 * scale)
+
+
+@pytest.mark.parametrize("name", ["tiny", "qwen3_4b", "qwen3_8b", "long"])
+def test_topk_configs(taps, name):
+    cfg = W.CONFIGS[name]
+    B = min(cfg.B, 2)
+    x = W.make_logits(cfg, B=B)
+    _check_topk(taps, x, cfg.K, torch.float32 if cfg.logits_dtype == "f32" else torch.bfloat16)
+
+
+@pytest.mark.slow
+def test_topk_batched_full(taps):
+    cfg = W.CONFIGS["batched"]
+    x = W.make_logits(cfg)
+    _check_topk(taps, x, cfg.K, torch.bfloat16)
+
+
+@pytest.mark.parametrize("V,K,B,L", [(1, 1, 1, 1), (7, 7, 1, 3), (2047, 5, 2, 2), (4099, 32, 1, 2),
+                                     (151937, 8, 1, 2), (100003, 16, 3, 5), (262143, 3, 1, 1)])
+def test_topk_ragged_sizes(taps, V, K, B, L):
+    rng = np.random.default_rng(V)
+    x = (rng.standard_normal((B, L, V)) * 4).astype(np.float32)
+    _check_topk(taps, x, K)
+    _check_topk(taps, W.round_to_bf16(x), K, torch.bfloat16)
+
+
+def test_topk_ties_and_minus_inf(taps):
+    rng = np.random.default_rng(3)
+    x = rng.integers(-4, 3, size=(2, 3, 30011)).astype(np.float32)     # heavy exact ties
+    x[0, 0, ::3] = -np.inf
+    x[1, 2, :] = 0.0
+    x[1, 2, 17] = -0.0
+    _check_topk(taps, x, 32)
+    _check_topk(taps, x, 1)
+
+
+def test_topk_strided_rows(taps):
+    """Rows with a stride that is not a multiple of 16 bytes take the scalar path."""
+    rng = np.random.default_rng(4)
+    V, pad = 5003, 3
+    full = (rng.standard_normal((2, 4, V + pad)) * 2).astype(np.float32)
+    xd = dt(full)[:, :, :V]
+    _check_topk(taps, full[:, :, :V], 8, x_dev=xd)
+
+
+# ---------------------------------------------------------------------------
+# Stage 2 (same inputs on both sides: the oracle's stage-1 results in f32)
+# ---------------------------------------------------------------------------
+
+def _stage1_inputs(cfg, B=None):
+    x = W.make_logits(cfg, B=B)
+    ids, logp, lse, ent = O.topk_marginals(x, cfg.K)
+    root = W.make_root_tokens(cfg, B=x.shape[0])
+    return x, ids, logp.astype(np.float32), ent.astype(np.float32), root
+
+
+@pytest.mark.parametrize("name,kind", [("tiny", "mlp"), ("tiny", "marginal"),
+                                       ("qwen3_8b", "mlp"), ("long", "mlp"),
+                                       ("qwen3_8b", "marginal")])
+def test_score_parity(taps, name, kind):
+    cfg = W.CONFIGS[name]
+    x, ids, logp, ent, root = _stage1_inputs(cfg, B=min(cfg.B, 2))
+    w = W.make_scorer_weights(cfg)
+    if kind == "mlp":
+        sp = taps.scorer_params("mlp", dt(w["packed"]), w["E"], w["H"], w["V"], w["max_depth"])
+    else:
+        sp = taps.scorer_params("marginal")
+    q = taps.taps_score_reach(dt(root), dt(ids), dt(logp), dt(ent), sp)
+    torch.cuda.synchronize()
+    ref = O.score_qcond(root, ids, logp, ent, kind, w)
+    np.testing.assert_allclose(host(q), ref, rtol=1e-5, atol=1e-7)
+
+
+# ---------------------------------------------------------------------------
+# Stage 3 (same q_cond on both sides: bit-exact)
+# ---------------------------------------------------------------------------
+
+SEL_KEYS = ("n_nodes", "parent", "depth", "token", "slot", "pos_id", "reach", "utility")
+
+
+def _check_select(taps, q, ids, root, ctx, l1, l2, tau, n_max):
+    out = taps.taps_select_subtree(dt(q), dt(ids), dt(root), dt(ctx), l1, l2, tau, n_max)
+    torch.cuda.synchronize()
+    ref = O.select_subtree(q, ids, root, ctx, l1, l2, tau, n_max)
+    for k in SEL_KEYS:
+        np.testing.assert_array_equal(host(out[k]), ref[k], err_msg=k)
+    return ref
+
+
+@pytest.mark.parametrize("name,n_max", [("tiny", 16), ("qwen3_8b", 32), ("qwen3_8b", 64),
+                                        ("qwen3_8b", 128), ("qwen3_8b", 256), ("long", 256),
+                                        ("qwen3_4b", 512)])
+def test_select_parity(taps, name, n_max):
+    cfg = W.CONFIGS[name]
+    x, ids, logp, ent, root = _stage1_inputs(cfg, B=min(cfg.B, 2))
+    w = W.make_scorer_weights(cfg)
+    q = O.score_qcond(root, ids, logp, ent, "mlp", w)
+    ctx = W.make_ctx_lens(cfg, B=x.shape[0])
+    _check_select(taps, q, ids, root, ctx, cfg.lambda1, cfg.lambda2, 0.0, n_max)
+
+
+def test_select_batched_requests(taps):
+    cfg = W.CONFIGS["batched"]
+    rng = np.random.default_rng(11)
+    B, L, K = 32, 16, 8
+    raw = rng.random((B, L, K, K)) ** 3 + 1e-3
+    q = (raw / raw.sum(-1, keepdims=True)).astype(np.float32)
+    q[:, 0, 1:] = 0
+    ids = np.stack([np.stack([rng.permutation(151936)[:K] for _ in range(L)]) for _ in range(B)])
+    ids = ids.astype(np.int32)
+    root = rng.integers(0, 151936, size=B).astype(np.int32)
+    ctx = W.make_ctx_lens(cfg)
+    _check_select(taps, q, ids, root, ctx, 1.0, 0.1, 0.0, 64)
+
+
+@pytest.mark.parametrize("tau", [1e-3, 2e-2, 0.3, 5.0])
+def test_select_adaptive_threshold(taps, tau):
+    cfg = W.CONFIGS["qwen3_8b"]
+    x, ids, logp, ent, root = _stage1_inputs(cfg, B=1)
+    q = O.score_qcond(root, ids, logp, ent, "marginal")
+    ref = _check_select(taps, q, ids, root, np.array([7], np.int32), 1.0, 0.1, tau, 256)
+    assert ref["n_nodes"][0] < 256 or tau < 1e-2
+
+
+def test_select_ties_chain_and_limits(taps):
+    rng = np.random.default_rng(5)
+    # exact ties everywhere: few distinct probabilities
+    L, K = 31, 32
+    raw = rng.choice([1.0, 2.0, 4.0], size=(1, L, K, K))
+    q = (raw / raw.sum(-1, keepdims=True)).astype(np.float32)
+    q[:, 0, 1:] = 0
+    ids = np.stack([rng.permutation(262143)[:K] for _ in range(L)])[None].astype(np.int32)
+    _check_select(taps, q, ids, np.array([5], np.int32), np.array([0], np.int32),
+                  1.0, 0.0, 0.0, 512)
+    _check_select(taps, q, ids, np.array([5], np.int32), np.array([0], np.int32),
+                  0.5, 0.25, 0.0, 300)
+    # K = 1: a chain (single-path verification)
+    q1 = np.ones((1, 12, 1, 1), np.float32)
+    ids1 = np.arange(12, dtype=np.int32).reshape(1, 12, 1)
+    ref = _check_select(taps, q1, ids1, np.array([3], np.int32), np.array([9], np.int32),
+                        1.0, 0.1, 0.0, 8)
+    assert ref["n_nodes"][0] == 8
+    # budget 1: the root only
+    ref = _check_select(taps, q1, ids1, np.array([3], np.int32), np.array([9], np.int32),
+                        1.0, 0.1, 0.0, 1)
+    assert ref["n_nodes"][0] == 1
+
+
+def test_select_underflowing_reach(taps):
+    """Tiny q_cond values make deep reach underflow to subnormals and zero."""
+    L, K = 20, 4
+    q = np.zeros((1, L, K, K), np.float32)
+    q[0, :, :, :] = np.array([1 - 3e-8, 1e-8, 1e-8, 1e-8], np.float32)
+    q[0, 0, 1:] = 0
+    q[0, 5:, :, 1:] = np.float32(1e-30)
+    ids = np.tile(np.arange(K, dtype=np.int32), (1, L, 1)) + 100
+    _check_select(taps, q, ids, np.array([1], np.int32), np.array([0], np.int32),
+                  1.0, 0.1, 0.0, 200)
+
+
+# ---------------------------------------------------------------------------
+# Stage 4
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("n_max", [1, 16, 33, 64, 256, 512])
+def test_mask_parity(taps, n_max):
+    rng = np.random.default_rng(n_max)
+    B = 3
+    parent = np.full((B, n_max), -1, np.int32)
+    n_nodes = np.array([n_max, max(1, n_max // 2), 1], np.int32)
+    for b in range(B):
+        for i in range(1, n_nodes[b]):
+            parent[b, i] = rng.integers(max(0, i - 20), i)
+    m = taps.taps_build_tree_mask(dt(parent), dt(n_nodes))
+    torch.cuda.synchronize()
+    ref = O.build_tree_mask(parent, n_nodes, n_max)
+    np.testing.assert_array_equal(host(m).view(np.uint32), ref)
+
+
+# ---------------------------------------------------------------------------
+# Stage 5
+# ---------------------------------------------------------------------------
+
+def _tree(rng, n_max, n, L=16):
+    parent = np.full((1, n_max), -1, np.int32)
+    depth = np.zeros(n, int)
+    for i in range(1, n):
+        cands = [j for j in range(i) if depth[j] < L]
+        parent[0, i] = rng.choice(cands)
+        depth[i] = depth[parent[0, i]] + 1
+    return parent
+
+
+def _attn_inputs(cfg, B, n_nodes, ctx, n_max, device_kv=False, seed=0):
+    rng = np.random.default_rng(seed)
+    parent = np.concatenate([_tree(rng, n_max, int(n)) for n in n_nodes])
+    mask = O.build_tree_mask(parent, n_nodes, n_max)
+    bt, num_pages = W.make_block_table(cfg, ctx, n_max)
+    if device_kv:
+        kc, vc = W.make_kv_torch(cfg, num_pages, 0, DEV)
+        q = W.make_q_torch(cfg, B, n_max, 0, DEV)
+    else:
+        kn, vn = W.make_kv_numpy(cfg, num_pages)
+        kc, vc = bf(kn), bf(vn)
+        q = bf(W.make_q_numpy(cfg, B, n_max))
+    return q, kc, vc, bt, mask
+
+
+def _run_attn(taps, q, kc, vc, bt, ctx, n_nodes, mask, status=None):
+    out, lse = taps.taps_tree_verify_attn(q, kc, vc, dt(bt), dt(ctx), dt(n_nodes),
+                                          dt(mask.view(np.int32)), int(ctx.max()),
+                                          want_lse=True, status=status)
+    torch.cuda.synchronize()
+    return out, lse
+
+
+def _f32(t):
+    return t.float().cpu().numpy()
+
+
+@pytest.mark.parametrize("name,n,ctx", [("tiny", 16, 512), ("tiny", 1, 512), ("tiny", 5, 0),
+                                        ("tiny", 13, 37), ("qwen3_8b", 64, 300),
+                                        ("qwen3_8b", 33, 1000)])
+def test_attention_parity_small(taps, name, n, ctx):
+    cfg = W.CONFIGS[name]
+    n_max = max(16, n)
+    ctx_a = np.array([ctx], np.int32)
+    nn = np.array([n], np.int32)
+    q, kc, vc, bt, mask = _attn_inputs(cfg, 1, nn, ctx_a, n_max)
+    out, lse = _run_attn(taps, q, kc, vc, bt, ctx_a, nn, mask)
+    ref, ref_lse = O.tree_verify_attn(_f32(q), _f32(kc), _f32(vc), bt, ctx_a, nn, mask)
+    assert np.abs(_f32(out) - ref).max() <= ATTN_ATOL
+    np.testing.assert_allclose(host(lse)[0, :n], ref_lse[0, :n], rtol=1e-4, atol=1e-4)
+    assert np.all(_f32(out)[0, n:] == 0)
+
+
+def _sampled_check(q, kc, vc, bt, ctx, nn, mask, out, rng, per_req=6):
+    """Oracle on sampled (request, node, head) rows, gathering the request's pages."""
+    B, n_max, Hq, D = q.shape
+    qh, kh, vh = _f32(q), None, None
+    o = _f32(out)
+    worst = 0.0
+    for b in range(B):
+        n = int(nn[b])
+        pages = bt[b][bt[b] >= 0]
+        kb = kc[torch.from_numpy(pages.astype(np.int64)).to(kc.device)].float().cpu().numpy()
+        vb = vc[torch.from_numpy(pages.astype(np.int64)).to(vc.device)].float().cpu().numpy()
+        bt_b = np.arange(len(pages), dtype=np.int32)[None]
+        rows = {(0, int(rng.integers(0, n)), int(rng.integers(0, Hq))) for _ in range(per_req)}
+        rows |= {(0, n - 1, Hq - 1), (0, 0, 0)}
+        ref, _ = O.tree_verify_attn(qh[b:b + 1], kb, vb, bt_b, ctx[b:b + 1], nn[b:b + 1],
+                                    mask[b:b + 1], only=rows)
+        for (_, i, h) in rows:
+            worst = max(worst, float(np.abs(o[b, i, h] - ref[0, i, h]).max()))
+        assert np.all(o[b, n:] == 0)
+    assert worst <= ATTN_ATOL, worst
+    return worst
+
+
+@pytest.mark.parametrize("name,n", [("qwen3_8b", 64), ("qwen3_8b", 256), ("qwen3_4b", 64)])
+def test_attention_full_size_sampled(taps, name, n):
+    cfg = W.CONFIGS[name]
+    ctx = W.make_ctx_lens(cfg)
+    nn = np.array([n], np.int32)
+    q, kc, vc, bt, mask = _attn_inputs(cfg, 1, nn, ctx, n, device_kv=True)
+    out, _ = _run_attn(taps, q, kc, vc, bt, ctx, nn, mask)
+    _sampled_check(q, kc, vc, bt, ctx, nn, mask, out, np.random.default_rng(1))
+
+
+@pytest.mark.slow
+@pytest.mark.parametrize("name", ["batched", "long"])
+def test_attention_batched_and_long_sampled(taps, name):
+    cfg = W.CONFIGS[name]
+    ctx = W.make_ctx_lens(cfg)
+    rng = np.random.default_rng(2)
+    nn = rng.integers(1, cfg.n_max + 1, size=cfg.B).astype(np.int32)
+    nn[0] = cfg.n_max
+    q, kc, vc, bt, mask = _attn_inputs(cfg, cfg.B, nn, ctx, cfg.n_max, device_kv=True)
+    out, _ = _run_attn(taps, q, kc, vc, bt, ctx, nn, mask)
+    _sampled_check(q, kc, vc, bt, ctx, nn, mask, out, rng, per_req=3)
+
+
+def test_attention_bad_page_sets_status(taps):
+    cfg = W.CONFIGS["tiny"]
+    ctx = np.array([200], np.int32)
+    nn = np.array([4], np.int32)
+    q, kc, vc, bt, mask = _attn_inputs(cfg, 1, nn, ctx, 16)
+    bt = bt.copy()
+    bt[0, 3] = kc.shape[0] + 5            # out of range: skipped and reported
+    status = torch.zeros(1, dtype=torch.int32, device=DEV)
+    out, _ = _run_attn(taps, q, kc, vc, bt, ctx, nn, mask, status=status)
+    assert int(status.item()) & taps.TAPS_DEVFAULT_PAGE
+    assert np.all(np.isfinite(_f32(out)))
+    status.zero_()
+    bt[0, 3] = 0
+    _run_attn(taps, q, kc, vc, bt, ctx, nn, mask, status=status)
+    assert int(status.item()) == 0
+
+
+# ---------------------------------------------------------------------------
+# Stage 6
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("seed", range(6))
+def test_accept_parity(taps, seed):
+    rng = np.random.default_rng(seed)
+    B, L, K, n_max = 4, 16, 4, 96
+    raw = rng.random((B, L, K, K)) + 0.05
+    q = (raw / raw.sum(-1, keepdims=True)).astype(np.float32)
+    q[:, 0, 1:] = 0
+    ids = rng.integers(0, 5, size=(B, L, K)).astype(np.int32)
+    for b in range(B):
+        for d in range(L):
+            ids[b, d] = rng.permutation(6)[:K]
+    sel = O.select_subtree(q, ids, np.zeros(B, np.int32), np.zeros(B, np.int32), 1.0, 0.1, 0.0,
+                           n_max)
+    y = rng.integers(0, 6, size=(B, L + 1)).astype(np.int32)
+    tt = W.target_tokens_for_tree(y, sel["depth"], sel["n_nodes"])
+    alen, nodes, bonus = taps.taps_accept(dt(sel["parent"]), dt(sel["token"]),
+                                          dt(sel["n_nodes"]), dt(tt), L)
+    torch.cuda.synchronize()
+    r = O.accept(sel["parent"], sel["token"], sel["n_nodes"], tt, L)
+    np.testing.assert_array_equal(host(alen), r[0])
+    np.testing.assert_array_equal(host(nodes), r[1])
+    np.testing.assert_array_equal(host(bonus), r[2])
+
+
+# ---------------------------------------------------------------------------
+# End to end through TapsRound
+# ---------------------------------------------------------------------------
+
+def _near_tie_valid(tree, q_ref, ids, L, K, lambda1, lambda2, rtol=1e-5):
+    """The GPU's tree is a valid greedy result under the oracle's q_cond, up to
+    a relative utility tolerance: no unselected child of the tree beats a
+    selected node by more than rtol."""
+    n = int(tree["n_nodes"])
+    paths = [()]
+    for i in range(1, n):
+        paths.append(paths[int(tree["parent"][i])] + (int(tree["slot"][i]),))
+    pset = set(paths)
+
+    def util(p):
+        return O.reach_of_path(q_ref.astype(np.float64), p) / (lambda1 + lambda2 * len(p))
+    sel_min = min(util(p) for p in paths[1:]) if n > 1 else np.inf
+    front_max = 0.0
+    for p in paths:
+        if len(p) < L:
+            for j in range(K):
+                c = p + (j,)
+                if c not in pset:
+                    front_max = max(front_max, util(c))
+    return front_max <= sel_min * (1 + rtol)
+
+
+@pytest.mark.parametrize("name,n_max", [("tiny", 16), ("qwen3_8b", 64), ("qwen3_8b", 256)])
+def test_round_end_to_end(taps, name, n_max):
+    cfg = W.CONFIGS[name]
+    x = W.make_logits(cfg)
+    root, ctx = W.make_root_tokens(cfg), W.make_ctx_lens(cfg)
+    w = W.make_scorer_weights(cfg)
+    bt, num_pages = W.make_block_table(cfg, ctx, n_max)
+    r = taps.TapsRound(B=cfg.B, L=cfg.L, V=cfg.V, K=cfg.K, n_max=n_max, Hq=cfg.Hq, Hkv=cfg.Hkv,
+                       D=cfg.D, max_ctx=int(ctx.max()), device=DEV,
+                       scorer_weights=dt(w["packed"]), emb_dim=w["E"], hidden=w["H"],
+                       lambda1=cfg.lambda1, lambda2=cfg.lambda2, tau=cfg.tau)
+    xd = dt(x).to(torch.float32 if cfg.logits_dtype == "f32" else torch.bfloat16)
+    r.select(xd, dt(root), dt(ctx))
+    torch.cuda.synchronize()
+    ids, logp, lse, ent = O.topk_marginals(x, cfg.K)
+    np.testing.assert_array_equal(host(r.ids), ids)
+    q_ref = O.score_qcond(root, ids, logp, ent, "mlp", w)
+    np.testing.assert_allclose(host(r.q_cond), q_ref, rtol=1e-4, atol=1e-6)
+    # topology: bit-exact given the GPU's own q_cond, near-tie valid under the oracle's
+    gq = host(r.q_cond)
+    ref = O.select_subtree(gq, ids, root, ctx, cfg.lambda1, cfg.lambda2, cfg.tau, n_max)
+    sel = {k: host(v) for k, v in r.sel.items()}
+    for k in SEL_KEYS:
+        np.testing.assert_array_equal(sel[k], ref[k], err_msg=k)
+    tree0 = {k: v[0] for k, v in sel.items()}
+    assert _near_tie_valid(tree0, q_ref[0], ids[0], cfg.L, cfg.K, cfg.lambda1, cfg.lambda2)
+    mask = O.build_tree_mask(sel["parent"], sel["n_nodes"], n_max)
+    np.testing.assert_array_equal(host(r.mask).view(np.uint32), mask)
+    # one verification layer
+    if cfg.D * cfg.Hq * n_max <= 128 * 32 * 256:
+        kn, vn = W.make_kv_numpy(cfg, num_pages)
+        qn = W.make_q_numpy(cfg, cfg.B, n_max)
+        out = torch.empty((cfg.B, n_max, cfg.Hq, cfg.D), dtype=torch.bfloat16, device=DEV)
+        r.verify_layer(bf(qn), bf(kn), bf(vn), dt(bt), dt(ctx), out)
+        torch.cuda.synchronize()
+        rows = {(0, i, h) for i in range(0, int(sel["n_nodes"][0]), 7) for h in (0, cfg.Hq - 1)}
+        o_ref, _ = O.tree_verify_attn(qn, kn, vn, bt, ctx, sel["n_nodes"], mask, only=rows)
+        o = _f32(out)
+        for (_, i, h) in rows:
+            assert np.abs(o[0, i, h] - o_ref[0, i, h]).max() <= ATTN_ATOL
+    y = W.make_target_sequence(cfg, x)
+    tt = W.target_tokens_for_tree(y, sel["depth"], sel["n_nodes"])
+    r.accept(dt(tt))
+    torch.cuda.synchronize()
+    a = O.accept(sel["parent"], sel["token"], sel["n_nodes"], tt, cfg.L)
+    np.testing.assert_array_equal(host(r.accept_len), a[0])
+    np.testing.assert_array_equal(host(r.accepted_nodes), a[1])
+    np.testing.assert_array_equal(host(r.bonus_tok), a[2])
