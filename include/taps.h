@@ -79,8 +79,13 @@ int taps_version(void);
  * topk_logp  [B, L, K] f32, out: logit - lse (full-vocabulary log-probability).
  * lse        [B, L] f32, out: log sum_v exp(logit_v).
  * entropy    [B, L] f32, out: -sum_v p_v log p_v in nats, full vocabulary.
- * ws         workspace of taps_topk_marginals_workspace_bytes(B, L, V, K).
- * Limits: 1 <= K <= min(32, V), 1 <= V <= 262143. Logits must be finite.
+ * ws         workspace of taps_topk_marginals_workspace_bytes(B, L, V, K); its
+ *            first 256 KiB hold per-row counters that must be zero before the
+ *            first call and that every call leaves at zero, so one zero-filled
+ *            workspace can serve calls of any shape on one stream.
+ * Limits: 1 <= K <= min(32, V), 1 <= V <= 262143. Logits may be -inf
+ * (probability 0, no entropy contribution) but not +inf or NaN, and every row
+ * needs at least K finite logits for the top-K to be meaningful.
  * ---------------------------------------------------------------------- */
 size_t taps_topk_marginals_workspace_bytes(int B, int L, int V, int K);
 int taps_topk_marginals(const void* logits, int dtype, int64_t row_stride,

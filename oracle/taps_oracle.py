@@ -77,7 +77,9 @@ def topk_marginals(logits: np.ndarray, K: int):
     Z = np.exp(x - m[..., None]).sum(axis=-1)
     lse = m + np.log(Z)
     p = np.exp(x - lse[..., None])
-    entropy = -(p * (x - lse[..., None])).sum(axis=-1)
+    # tokens of probability 0 (logit -inf) contribute 0 (the 0 log 0 = 0 convention)
+    logp_all = np.where(p > 0, x - lse[..., None], 0.0)
+    entropy = -(p * logp_all).sum(axis=-1)
     ids = np.empty((B, L, K), np.int32)
     for b in range(B):
         for d in range(L):

@@ -47,15 +47,21 @@ struct WsLayout {
   size_t stats, keys, tickets, total;
 };
 
+// The per-row tickets always sit in a fixed region at the start of the
+// workspace, sized for the largest row count, so that a workspace reused by
+// calls of different shapes never finds partial records where a later call
+// keeps its counters. Every call leaves its tickets at zero.
+constexpr size_t kTicketRegion = sizeof(unsigned) * 65536;
+
 WsLayout ws_layout(const Plan& p) {
   WsLayout w;
   size_t o = 0;
+  w.tickets = o;
+  o = kTicketRegion;
   w.stats = o;
   o = align_up(o + sizeof(float4) * p.rows * p.chunks, 256);
   w.keys = o;
   o = align_up(o + sizeof(uint64_t) * p.rows * p.chunks * p.kp, 256);
-  w.tickets = o;
-  o = align_up(o + sizeof(unsigned) * p.rows, 256);
   w.total = o;
   return w;
 }

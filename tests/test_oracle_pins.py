@@ -61,6 +61,20 @@ def test_marginals_two_level_closed_form(a, A):
     assert ids[0, 0].tolist() == expect
 
 
+def test_marginals_minus_inf_is_probability_zero():
+    """Masked tokens (logit -inf) have probability 0 and add nothing to the
+    entropy: the statistics equal those of the row without them."""
+    V = 300
+    x = np.random.default_rng(8).standard_normal((1, 1, V))
+    xm = x.copy()
+    xm[0, 0, ::2] = -np.inf
+    ids, logp, lse, ent = O.topk_marginals(xm, 4)
+    ids2, logp2, lse2, ent2 = O.topk_marginals(x[:, :, 1::2], 4)
+    assert lse[0, 0] == pytest.approx(lse2[0, 0], rel=1e-13)
+    assert ent[0, 0] == pytest.approx(ent2[0, 0], rel=1e-12)
+    assert (ids[0, 0] == 2 * ids2[0, 0] + 1).all()
+
+
 def test_topk_brute_force_rank_with_ties():
     rng = np.random.default_rng(1)
     x = rng.integers(-3, 4, size=(2, 3, 50)).astype(np.float32)   # many exact ties
