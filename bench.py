@@ -1,0 +1,478 @@
+"""Benchmark: TAPS rounds per second (select + tree verify) on one GB300.
+
+One step = one full TAPS round over one batch of synthetic input, all stages
+of Sec. 4.1 on the GPU: top-K marginals, scoring, selection, mask, tree
+verification attention for every layer of the target, acceptance. The round
+is captured as three CUDA graphs (stages 1-4, the per-layer attention calls,
+stage 6) and replayed; CUDA events between the graphs time the attention
+stage live for the roofline figure.
+
+Workload (default): Qwen3-8B shape, batch 1, draft block L=16, vocab 151936,
+bf16 drafter logits (Zipf s=1.1 with position temperature 0.6 -> 1.4), top-K 8,
+node budget 64, 36 layers x (32 q heads, 8 KV heads, head dim 128), context
+4096, paged bf16 KV cache with 16-token pages, a distinct cache per layer.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+``--impl reference`` times the plain CPU oracle (the method written from the
+paper) on the host cores on a bounded sample of the same workload.
+Multi-GPU: the round does not shard (replicas only); under torchrun every
+rank runs its own replica and rank 0 reports the aggregate.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+FALLBACK_HBM_GBS = 6800.0
+FALLBACK_BF16_TFLOPS = 1900.0
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), float(d["bf16_tflops"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, FALLBACK_BF16_TFLOPS, "fallback"
+
+
+def workload_config(name, n_max, layers):
+    import workloads as W
+    cfg = W.CONFIGS[name]
+    return cfg.with_(n_max=n_max, layers=layers)
+
+
+def attn_bytes_flops(cfg, ctx, n_nodes, depth):
+    """Algorithmic bytes and flops of one attention layer (every request):
+    K and V of the visible context plus the tree nodes, Q read and O write;
+    flops count QK^T and PV over the context and the ancestor-or-self pairs."""
+    byt, fl = 0, 0
+    for b in range(len(ctx)):
+        C, n = int(ctx[b]), int(n_nodes[b])
+        byt += (C + n) * cfg.Hkv * cfg.D * 2 * 2 + 2 * n * cfg.Hq * cfg.D * 2
+        pairs = n * C + int(sum(int(d) + 1 for d in depth[b][:n]))
+        fl += 4 * cfg.Hq * cfg.D * pairs
+    return byt, fl
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled during the timed region."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        out, _ = self.proc.communicate(timeout=10)
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.strip().splitlines():
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx.append(float(parts[2]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(nm)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# CPU baseline: the oracle as it stands, on a bounded sample of the workload
+# ---------------------------------------------------------------------------
+
+def oracle_step(cfg, inp, sample_layers):
+    """One oracle round: stages 1-4 and 6 on the whole batch, stage 5 on
+    ``sample_layers`` of the cfg.layers layers; returns seconds scaled to the
+    full round."""
+    from oracle import taps_oracle as O
+    t0 = time.perf_counter()
+    ids, logp, lse, ent = O.topk_marginals(inp["logits"], cfg.K)
+    q = O.score_qcond(inp["root"], ids, logp, ent, "mlp", inp["w"])
+    sel = O.select_subtree(q, ids, inp["root"], inp["ctx"], cfg.lambda1, cfg.lambda2, cfg.tau,
+                           cfg.n_max)
+    mask = O.build_tree_mask(sel["parent"], sel["n_nodes"], cfg.n_max)
+    import workloads as W
+    tt = W.target_tokens_for_tree(inp["y"], sel["depth"], sel["n_nodes"])
+    O.accept(sel["parent"], sel["token"], sel["n_nodes"], tt, cfg.L)
+    t1 = time.perf_counter()
+    for _ in range(sample_layers):
+        O.tree_verify_attn(inp["q"], inp["k"], inp["v"], inp["bt"], inp["ctx"], sel["n_nodes"],
+                           mask)
+    t2 = time.perf_counter()
+    per_layer = (t2 - t1) / max(sample_layers, 1)
+    return (t1 - t0) + cfg.layers * per_layer, t2 - t0
+
+
+def oracle_inputs(cfg):
+    import workloads as W
+    logits = W.make_logits(cfg)
+    ctx = W.make_ctx_lens(cfg)
+    bt, num_pages = W.make_block_table(cfg, ctx)
+    k, v = W.make_kv_numpy(cfg, num_pages)
+    return dict(logits=logits, root=W.make_root_tokens(cfg), ctx=ctx, bt=bt, k=k, v=v,
+                q=W.make_q_numpy(cfg, cfg.B, cfg.n_max), w=W.make_scorer_weights(cfg),
+                y=W.make_target_sequence(cfg, logits))
+
+
+def cpu_child(args):
+    """Runs in a fresh single-threaded process: prints the oracle timing JSON."""
+    cfg = workload_config(args.workload, args.n_max, args.layers)
+    inp = oracle_inputs(cfg)
+    steps, warm = args.steps, args.warmup
+    for _ in range(warm):
+        oracle_step(cfg, inp, args.sample_layers)
+    scaled, wall = [], []
+    for _ in range(steps):
+        s, w = oracle_step(cfg, inp, args.sample_layers)
+        scaled.append(s)
+        wall.append(w)
+    print(json.dumps({"scaled_s": scaled, "wall_s": wall}))
+
+
+def run_cpu_baseline(args, steps, warmup, sample_layers):
+    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1",
+               CUDA_VISIBLE_DEVICES="")
+    cmd = [sys.executable, os.path.abspath(__file__), "--cpu-child", "--workload", args.workload,
+           "--n-max", str(args.n_max), "--layers", str(args.layers), "--steps", str(steps),
+           "--warmup", str(warmup), "--sample-layers", str(sample_layers)]
+    r = subprocess.run(cmd, env=env, capture_output=True, text=True)
+    if r.returncode != 0:
+        raise RuntimeError(f"cpu baseline child failed:\n{r.stderr[-2000:]}")
+    return json.loads(r.stdout.strip().splitlines()[-1])
+
+
+def sample_desc(cfg, sample_layers):
+    return (f"oracle stages 1-4 and 6 on the whole round, stage 5 on {sample_layers} of "
+            f"{cfg.layers} layers (timed, then scaled to {cfg.layers} layers)")
+
+
+# ---------------------------------------------------------------------------
+# the GPU arm
+# ---------------------------------------------------------------------------
+
+def dist_setup(args):
+    import torch
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        dist.init_process_group(backend)
+    return world, rank, local
+
+
+def max_over_ranks(x: float, world: int, device=None) -> float:
+    """Largest value of x over all ranks (the job's wall time is the slowest rank's)."""
+    if world <= 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def run_ours(args):
+    import numpy as np
+    import torch
+
+    import __graft_entry__
+    __graft_entry__.build()
+    import paper_2606_00487_gb300 as taps
+    import workloads as W
+
+    world, rank, local = dist_setup(args)
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    cfg = workload_config(args.workload, args.n_max, args.layers)
+
+    # ---- inputs (seeded, synthetic; KV and Q drawn on the device)
+    logits_h = W.make_logits(cfg)
+    root_h, ctx_h = W.make_root_tokens(cfg), W.make_ctx_lens(cfg)
+    w = W.make_scorer_weights(cfg)
+    bt_h, num_pages = W.make_block_table(cfg, ctx_h)
+    y = W.make_target_sequence(cfg, logits_h)
+    ldt = torch.bfloat16 if cfg.logits_dtype == "bf16" else torch.float32
+    logits = torch.from_numpy(logits_h).to(dev).to(ldt)
+    root, ctx = torch.from_numpy(root_h).to(dev), torch.from_numpy(ctx_h).to(dev)
+    bt = torch.from_numpy(bt_h).to(dev)
+    layers = []
+    for layer in range(cfg.layers):
+        kc, vc = W.make_kv_torch(cfg, num_pages, layer, dev)
+        q = W.make_q_torch(cfg, cfg.B, cfg.n_max, layer, dev)
+        layers.append((q, kc, vc, bt))
+    outs = [torch.empty_like(layers[0][0]) for _ in range(cfg.layers)]
+
+    r = taps.TapsRound(B=cfg.B, L=cfg.L, V=cfg.V, K=cfg.K, n_max=cfg.n_max, Hq=cfg.Hq,
+                       Hkv=cfg.Hkv, D=cfg.D, max_ctx=int(ctx_h.max()), device=dev,
+                       scorer_weights=torch.from_numpy(w["packed"]).to(dev), emb_dim=w["E"],
+                       hidden=w["H"], lambda1=cfg.lambda1, lambda2=cfg.lambda2, tau=cfg.tau)
+    # the stand-in target model's greedy tokens depend on the (deterministic) tree
+    r.select(logits, root, ctx)
+    torch.cuda.synchronize()
+    sel_h = {k: v.cpu().numpy() for k, v in r.sel.items()}
+    tt_h = W.target_tokens_for_tree(y, sel_h["depth"], sel_h["n_nodes"])
+    target = torch.from_numpy(tt_h).to(dev)
+
+    # ---- capture the round as three graphs
+    s = torch.cuda.Stream(device=dev)
+    s.wait_stream(torch.cuda.current_stream(dev))
+    with torch.cuda.stream(s):
+        for _ in range(2):
+            r.run(logits, root, ctx, layers, outs, target)
+    torch.cuda.current_stream(dev).wait_stream(s)
+    torch.cuda.synchronize()
+    g_pre, g_attn, g_post = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g_pre, stream=s):
+        r.select(logits, root, ctx)
+    with torch.cuda.graph(g_attn, stream=s):
+        for (q, kc, vc, b_t), o in zip(layers, outs):
+            r.verify_layer(q, kc, vc, b_t, ctx, o)
+    with torch.cuda.graph(g_post, stream=s):
+        r.accept(target)
+    torch.cuda.synchronize()
+
+    stream = torch.cuda.current_stream(dev)
+
+    def step(ev_a=None, ev_b=None):
+        g_pre.replay()
+        if ev_a is not None:
+            ev_a.record(stream)
+        g_attn.replay()
+        if ev_b is not None:
+            ev_b.record(stream)
+        g_post.replay()
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+
+    clocks = ClockSampler(local)
+    clocks.start()
+    time.sleep(0.3)
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(args.steps)]
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier(world)
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for k in range(args.steps):
+        step(*evs[k])
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier(world)
+    elapsed_ms = e0.elapsed_time(e1)
+    attn_ms = sum(a.elapsed_time(b) for a, b in evs) / args.steps
+    clk = clocks.stop()
+    elapsed_ms = max_over_ranks(elapsed_ms, world, dev)
+    status = int(r.status.item())
+    assert status == 0, f"device fault status {status}"
+
+    # ---- select + one-layer round (stages 1-4, one attention layer, stage 6)
+    g_one = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g_one, stream=s):
+        r.select(logits, root, ctx)
+        q0, k0, v0, b0 = layers[0]
+        r.verify_layer(q0, k0, v0, b0, ctx, outs[0])
+        r.accept(target)
+    for _ in range(3):
+        g_one.replay()
+    torch.cuda.synchronize()
+    f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    reps = max(args.steps, 20)
+    f0.record(stream)
+    for _ in range(reps):
+        g_one.replay()
+    f1.record(stream)
+    torch.cuda.synchronize()
+    one_layer_us = f0.elapsed_time(f1) / reps * 1e3
+
+    # ---- end to end through the public API with host buffers
+    e2e = None
+    if not args.no_e2e:
+        pin = lambda t: t.cpu().pin_memory()
+        logits_pin = pin(logits)
+        q_pin = [pin(q) for (q, _, _, _) in layers]
+        target_pin = pin(target)
+        res_pin = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
+                   for t in (r.sel["n_nodes"], r.accept_len, r.accepted_nodes, r.bonus_tok)]
+        h2d = (logits_pin.numel() * logits_pin.element_size()
+               + sum(t.numel() * t.element_size() for t in q_pin)
+               + target_pin.numel() * target_pin.element_size())
+        d2h = sum(t.numel() * t.element_size() for t in res_pin)
+
+        def e2e_step():
+            logits.copy_(logits_pin, non_blocking=True)
+            for (q, _, _, _), qp in zip(layers, q_pin):
+                q.copy_(qp, non_blocking=True)
+            target.copy_(target_pin, non_blocking=True)
+            step()
+            for dst, src in zip(res_pin, (r.sel["n_nodes"], r.accept_len, r.accepted_nodes,
+                                          r.bonus_tok)):
+                dst.copy_(src, non_blocking=True)
+            stream.synchronize()
+
+        for _ in range(args.warmup):
+            e2e_step()
+        barrier(world)
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for _ in range(args.steps):
+            e2e_step()
+        t_e2e = max_over_ranks(time.perf_counter() - t0, world, dev)
+        e2e = {"value": world * args.steps / t_e2e, "unit": "rounds/s",
+               "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}
+
+    # ---- roofline of the attention stage (dominant kernel)
+    hbm, bf16, src = load_peaks()
+    byt, fl = attn_bytes_flops(cfg, ctx_h, sel_h["n_nodes"], sel_h["depth"])
+    per_launch_s = attn_ms / cfg.layers / 1e3
+    achieved_gbs = byt / per_launch_s / 1e9
+    achieved_tf = fl / per_launch_s / 1e12
+    traffic = None
+    tp = os.path.join(ROOT, "profiles", "attn_traffic.json")
+    if os.path.exists(tp):
+        try:
+            t = json.load(open(tp))
+            if t.get("workload") == cfg.name and t.get("n_max") == cfg.n_max:
+                traffic = t.get("bytes_per_launch")
+        except Exception:
+            traffic = None
+    roofline = {"bound": "hbm", "achieved": round(achieved_gbs, 1), "peak": hbm, "unit": "GB/s",
+                "frac": round(achieved_gbs / hbm, 4), "traffic": traffic,
+                "peak_source": src, "kernel": "taps_tree_verify_attn (one layer)",
+                "algorithmic_bytes_per_launch": byt, "avg_launch_us": round(per_launch_s * 1e6, 2),
+                "tensor_tflops": round(achieved_tf, 1),
+                "tensor_frac": round(achieved_tf / bf16, 4)}
+
+    launches = args.steps * (r.launches_per_select + cfg.layers * r.launches_per_layer + 1)
+    line = {
+        "metric": "TAPS rounds/sec (select+tree verify) at Qwen3-8B shape, 1 GB300; % HBM roofline",
+        "value": round(world * args.steps / (elapsed_ms / 1e3), 2),
+        "unit": "rounds/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(elapsed_ms / args.steps, 4),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded; shapes of the Qwen3-8B round, no weights or datasets)",
+        "config": {"workload": f"{cfg.name}: B={cfg.B} L={cfg.L} V={cfg.V} K={cfg.K} "
+                               f"n_max={cfg.n_max} layers={cfg.layers} Hq={cfg.Hq} Hkv={cfg.Hkv} "
+                               f"D={cfg.D} ctx={cfg.ctx} page={cfg.page}",
+                   "global_batch": cfg.B, "seq_len": int(ctx_h.max()), "parallelism": "replicas",
+                   "l2": "inputs larger than L2: 36 distinct KV layers, 0.6 GB per step",
+                   "n_nodes": int(sel_h["n_nodes"][0]),
+                   "select_plus_one_layer_round_us": round(one_layer_us, 2),
+                   "attention_stage_us_per_round": round(attn_ms * 1e3, 2)},
+        "roofline": roofline,
+        "e2e": e2e,
+        "gpu_launches": launches,
+        "clocks": clk,
+    }
+    if rank == 0 and not args.no_cpu_baseline:
+        cb = run_cpu_baseline(args, steps=1, warmup=0, sample_layers=args.sample_layers)
+        line["cpu_baseline"] = {"value": round(1.0 / cb["scaled_s"][0], 4), "unit": "rounds/s",
+                                "cores": 1, "kind": "oracle",
+                                "sample": sample_desc(cfg, args.sample_layers)
+                                + f"; wall {cb['wall_s'][0]:.1f} s"}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def run_reference(args):
+    """The oracle arm: rank 0 times the CPU oracle; other ranks exit."""
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    if rank != 0:
+        return
+    cfg = workload_config(args.workload, args.n_max, args.layers)
+    cb = run_cpu_baseline(args, steps=args.steps, warmup=args.warmup, sample_layers=1)
+    total = sum(cb["scaled_s"])
+    value = args.steps / total
+    line = {
+        "impl": "reference",
+        "metric": "TAPS rounds/sec (select+tree verify) at Qwen3-8B shape, 1 GB300; % HBM roofline",
+        "value": round(value, 5), "unit": "rounds/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(total / args.steps * 1e3, 2),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic (seeded; shapes of the Qwen3-8B round, no weights or datasets)",
+        "config": {"workload": f"{cfg.name}: B={cfg.B} L={cfg.L} V={cfg.V} K={cfg.K} "
+                               f"n_max={cfg.n_max} layers={cfg.layers} Hq={cfg.Hq} Hkv={cfg.Hkv} "
+                               f"D={cfg.D} ctx={cfg.ctx} page={cfg.page}",
+                   "global_batch": cfg.B, "seq_len": cfg.ctx if isinstance(cfg.ctx, int) else None,
+                   "parallelism": "none (host CPU)"},
+        "cpu_baseline": {"value": round(value, 5), "unit": "rounds/s", "cores": 1,
+                         "kind": "oracle", "sample": sample_desc(cfg, 1) + " per step"},
+        "e2e": {"value": round(value, 5), "unit": "rounds/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="qwen3_8b")
+    ap.add_argument("--n-max", type=int, default=64)
+    ap.add_argument("--layers", type=int, default=36)
+    ap.add_argument("--sample-layers", type=int, default=3)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-child", action="store_true", help=argparse.SUPPRESS)
+    args = ap.parse_args()
+    if args.warmup < 3 and not args.cpu_child:
+        args.warmup = 3
+    if args.cpu_child:
+        cpu_child(args)
+    elif args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()
