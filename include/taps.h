@@ -94,6 +94,36 @@ int taps_topk_marginals(const void* logits, int dtype, int64_t row_stride,
                         void* ws, size_t ws_bytes, void* stream);
 
 /* ------------------------------------------------------------------------
+ * taps_topk_marginals_noalloc - the same computation and outputs as
+ * taps_topk_marginals, for callers that cannot allocate device memory. The
+ * paper has no counterpart: this is a deployment convenience of this library.
+ *
+ * Who needs it: a serving engine that reserved all of device memory for its KV
+ * cache at start-up, a plugin running inside a host framework that owns every
+ * device allocation, or a decode loop that cannot afford the device-wide
+ * synchronisation cudaMalloc may cause. The caller still passes inputs and
+ * outputs; the partial records live in a fixed array of
+ * TAPS_NOALLOC_SCRATCH_BYTES (2 MiB) of device memory inside the library,
+ * which every GPU that loads the library holds until the process exits.
+ * Nothing is allocated or freed by this call.
+ *
+ * The first call on each device looks up that array's device address
+ * (cudaGetSymbolAddress, with the caller's current device); make that first
+ * call before any stream capture. Each call clears the counters it uses before
+ * its kernel runs. Every call shares the one array per device, so calls that
+ * overlap on the GPU (different streams, or different host threads without
+ * ordering) race: serialise them.
+ * Limits: B * L <= TAPS_NOALLOC_MAX_ROWS (4096); beyond it the call returns
+ * TAPS_ERR_UNSUPPORTED and launches nothing. Other limits as above.
+ * ---------------------------------------------------------------------- */
+#define TAPS_NOALLOC_MAX_ROWS 4096
+#define TAPS_NOALLOC_SCRATCH_BYTES (2u * 1024u * 1024u)
+int taps_topk_marginals_noalloc(const void* logits, int dtype, int64_t row_stride,
+                                int B, int L, int V, int K,
+                                int32_t* topk_ids, float* topk_logp, float* lse,
+                                float* entropy, void* stream);
+
+/* ------------------------------------------------------------------------
  * taps_score_reach - Sec. 4.2, Eq. 1 and Algorithm 1: for every parent of
  * the candidate trie, q_cond(parent -> child) = softmax over the K siblings
  * of the scorer logit of each edge.

@@ -280,3 +280,34 @@ def taps_accept(parent, token, n_nodes, target_tok, L, out=None, stream=None):
                          L, _ptr(alen), _ptr(nodes), _ptr(bonus), _stream(stream, dev))
     _check("taps_accept", st)
     return alen, nodes, bonus
+
+
+# ---------------------------------------------------------------------------
+# allocation-free variant of stage 1 (no counterpart in the paper)
+# ---------------------------------------------------------------------------
+
+lib.taps_topk_marginals_noalloc.argtypes = [_P, _I, _I64, _I, _I, _I, _I, _P, _P, _P, _P, _P]
+lib.taps_topk_marginals_noalloc.restype = _I
+
+
+def taps_topk_marginals_noalloc(logits: torch.Tensor, K: int, out, stream=None):
+    """Stage 1 for callers that cannot allocate device memory: the library
+    keeps its partial records in a fixed 2 MiB device array instead of a
+    workspace. ``out`` = (ids, logp, lse, entropy) must be preallocated by the
+    caller. Calls that overlap on the GPU share that array and race."""
+    if logits.dtype not in (torch.float32, torch.bfloat16) or not logits.is_cuda:
+        raise TypeError("logits must be a CUDA float32 or bfloat16 tensor")
+    B, L, V = logits.shape
+    if logits.stride(2) != 1 or logits.stride(0) != L * logits.stride(1):
+        raise ValueError("logits rows must be unit-stride with a uniform row stride")
+    ids, logp, lse, ent = out
+    _need(ids, torch.int32, (B, L, K), "ids")
+    _need(logp, torch.float32, (B, L, K), "logp")
+    _need(lse, torch.float32, (B, L), "lse")
+    _need(ent, torch.float32, (B, L), "entropy")
+    dtype = TAPS_F32 if logits.dtype == torch.float32 else TAPS_BF16
+    st = lib.taps_topk_marginals_noalloc(_ptr(logits), dtype, logits.stride(1), B, L, V, K,
+                                         _ptr(ids), _ptr(logp), _ptr(lse), _ptr(ent),
+                                         _stream(stream, logits.device))
+    _check("taps_topk_marginals_noalloc", st)
+    return ids, logp, lse, ent

@@ -11,6 +11,7 @@
 // atomic ticket, reset after use) merges the partials and writes the row's
 // outputs. No CTA waits on another.
 #include <algorithm>
+#include <mutex>
 
 #include "common.cuh"
 
@@ -377,6 +378,86 @@ extern "C" int taps_topk_marginals(const void* logits, int dtype, int64_t row_st
   const int vec_ok = aligned(logits, 16) && (row_stride * esz) % 16 == 0;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   char* wsc = static_cast<char*>(ws);
+  if (dtype == TAPS_F32)
+    dispatch_kp<float>(p.kp, logits, row_stride, p, V, K, vec_ok, topk_ids, topk_logp, lse,
+                       entropy, wsc, w, s);
+  else
+    dispatch_kp<__nv_bfloat16>(p.kp, logits, row_stride, p, V, K, vec_ok, topk_ids, topk_logp,
+                               lse, entropy, wsc, w, s);
+  return launch_status();
+}
+
+// ---------------------------------------------------------------------------
+// Allocation-free variant of taps_topk_marginals.
+//
+// Some callers cannot call cudaMalloc: a serving engine that reserved all of
+// device memory for its KV cache at start-up, a plugin running inside a host
+// framework that owns every device allocation, or a decode loop that cannot
+// afford the device-wide synchronisation an allocation may cause. This entry
+// point takes inputs and outputs from the caller and keeps its partial records
+// in a fixed array in device memory that belongs to this library.
+//
+// The array below is a file-scope __device__ symbol: every GPU that loads the
+// library holds it until the process exits. In host code its name is only a
+// host-side stand-in, never a device address, so the host looks the device
+// address up with cudaGetSymbolAddress, once per device, with that device
+// current, and passes that address to the kernel.
+// ---------------------------------------------------------------------------
+namespace taps {
+namespace {
+
+constexpr size_t kNoAllocTicketBytes = sizeof(unsigned) * TAPS_NOALLOC_MAX_ROWS;
+
+static __device__ __align__(256) unsigned char g_topk_scratch[TAPS_NOALLOC_SCRATCH_BYTES];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_scratch_mutex;
+void* g_scratch_ptr[kMaxDevices] = {};
+
+// Device address of g_topk_scratch on the current device (set up on first use).
+int scratch_for_current_device(void** out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return TAPS_ERR_CUDA;
+  std::lock_guard<std::mutex> lock(g_scratch_mutex);
+  if (!g_scratch_ptr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_topk_scratch) != cudaSuccess || !p) return TAPS_ERR_CUDA;
+    g_scratch_ptr[dev] = p;
+  }
+  *out = g_scratch_ptr[dev];
+  return TAPS_OK;
+}
+
+}  // namespace
+}  // namespace taps
+
+extern "C" int taps_topk_marginals_noalloc(const void* logits, int dtype, int64_t row_stride,
+                                           int B, int L, int V, int K, int32_t* topk_ids,
+                                           float* topk_logp, float* lse, float* entropy,
+                                           void* stream) {
+  if (!logits || !topk_ids || !topk_logp || !lse || !entropy) return TAPS_ERR_INVALID_ARG;
+  if (B <= 0 || L <= 0 || V <= 0 || K <= 0 || row_stride < V) return TAPS_ERR_INVALID_ARG;
+  if (dtype != TAPS_F32 && dtype != TAPS_BF16) return TAPS_ERR_INVALID_ARG;
+  if (K > TAPS_MAX_K || K > V || V > TAPS_MAX_V) return TAPS_ERR_UNSUPPORTED;
+  if (static_cast<int64_t>(B) * L > TAPS_NOALLOC_MAX_ROWS) return TAPS_ERR_UNSUPPORTED;
+  Plan p = make_plan(B, L, V, K);
+  // layout inside the fixed array: tickets, then the partial statistics, then keys
+  WsLayout w;
+  w.tickets = 0;
+  w.stats = kNoAllocTicketBytes;
+  w.keys = align_up(w.stats + sizeof(float4) * p.rows * p.chunks, 256);
+  w.total = align_up(w.keys + sizeof(uint64_t) * p.rows * p.chunks * p.kp, 256);
+  if (w.total > TAPS_NOALLOC_SCRATCH_BYTES) return TAPS_ERR_UNSUPPORTED;
+  void* scratch = nullptr;
+  int st = scratch_for_current_device(&scratch);
+  if (st != TAPS_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  // the tickets must start at zero; clear the ones this call uses
+  if (p.chunks > 1 && cudaMemsetAsync(scratch, 0, sizeof(unsigned) * p.rows, s) != cudaSuccess)
+    return TAPS_ERR_CUDA;
+  const size_t esz = dtype == TAPS_F32 ? 4 : 2;
+  const int vec_ok = aligned(logits, 16) && (row_stride * esz) % 16 == 0;
+  char* wsc = static_cast<char*>(scratch);
   if (dtype == TAPS_F32)
     dispatch_kp<float>(p.kp, logits, row_stride, p, V, K, vec_ok, topk_ids, topk_logp, lse,
                        entropy, wsc, w, s);
