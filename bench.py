@@ -239,6 +239,7 @@ def run_ours(args):
     layers = []
     for layer in range(cfg.layers):
         kc, vc = W.make_kv_torch(cfg, num_pages, layer, dev)
+        kc, vc = taps.taps_pack_kv_pages(kc), taps.taps_pack_kv_pages(vc)   # TAPS page layout
         q = W.make_q_torch(cfg, cfg.B, cfg.n_max, layer, dev)
         layers.append((q, kc, vc, bt))
     outs = [torch.empty_like(layers[0][0]) for _ in range(cfg.layers)]

@@ -54,7 +54,7 @@ typedef enum taps_status {
 
 enum { TAPS_F32 = 0, TAPS_BF16 = 1 };
 enum { TAPS_SCORER_MARGINAL = 0, TAPS_SCORER_MLP = 1 };
-enum { TAPS_DEVFAULT_PAGE = 1 };
+enum { TAPS_DEVFAULT_PAGE = 1, TAPS_DEVFAULT_TIMEOUT = 2 };
 
 /* Limits (TAPS_ERR_UNSUPPORTED beyond them). */
 #define TAPS_MAX_K 32
@@ -212,18 +212,23 @@ int taps_build_tree_mask(const int32_t* parent, const int32_t* n_nodes, int B, i
  * tree positions ctx_len[b] + j with bit j set in mask row i.
  *
  * q        [B, n_max, Hq, D] bf16 (post-RoPE queries of the tree nodes).
- * k_cache, v_cache [num_pages, Hkv, page_size, D] bf16. Logical position t
- *          of request b lives in page block_table[b * max_pages + t / page_size],
- *          row t % page_size. Tree node j's K/V must already sit at logical
- *          position ctx_len[b] + j, so pages must cover ctx_len[b] + n_nodes[b].
+ * k_cache, v_cache [num_pages, Hkv, page_size, D] bf16 blocks in the TAPS page
+ *          layout (taps_pack_kv_pages). Logical position t of request b lives
+ *          in page block_table[b * max_pages + t / page_size], row t % page_size.
+ *          Tree node j's K/V must already sit at logical position ctx_len[b] + j,
+ *          so pages must cover ctx_len[b] + n_nodes[b].
  * out      [B, n_max, Hq, D] bf16, out; rows i >= n_nodes[b] are written as 0.
  * lse_out  [B, n_max, Hq] f32, out, nullable: natural-log softmax denominator.
  * max_ctx  host upper bound of ctx_len[b] (sizes the split of the context).
- * ws       workspace of taps_tree_verify_attn_workspace_bytes(...).
+ * ws       unused (the chunks of a long context are combined on chip, inside
+ *          a thread-block cluster); taps_tree_verify_attn_workspace_bytes()
+ *          returns 0 and ws may be NULL.
  * status   device int32, nullable: TAPS_DEVFAULT_PAGE is ORed in when a page
  *          id is outside [0, num_pages); that page is then skipped.
- * Limits: D in {64, 128}, page_size == 16, Hq % Hkv == 0, Hq / Hkv <= 8,
- *         n_max <= 512.
+ *          TAPS_DEVFAULT_TIMEOUT is ORed in if an internal pipeline wait
+ *          exceeds its bound (about 2 s); the outputs are then undefined.
+ * Limits: D in {64, 128}, page_size == 16, Hq / Hkv in {1, 2, 4, 8},
+ *         n_max <= 512, max_ctx + n_max <= 65536.
  * ---------------------------------------------------------------------- */
 size_t taps_tree_verify_attn_workspace_bytes(int B, int n_max, int Hq, int Hkv, int D,
                                              int max_ctx);
@@ -233,6 +238,27 @@ int taps_tree_verify_attn(const void* q, const void* k_cache, const void* v_cach
                           int B, int n_max, int Hq, int Hkv, int D, int page_size, float scale,
                           int max_ctx, void* out, float* lse_out,
                           void* ws, size_t ws_bytes, int32_t* status, void* stream);
+
+/* ------------------------------------------------------------------------
+ * taps_pack_kv_pages / taps_unpack_kv_pages - the paged KV cache layout that
+ * taps_tree_verify_attn reads (Sec. 4.1 stage 3 verifies the tree against the
+ * target's KV cache; the paper fixes no layout, this one is the library's).
+ *
+ * The cache is [num_pages][Hkv] blocks of 16 tokens x D bf16 values (D in
+ * {64, 128}), 16 * D * 2 bytes each, in the same block order as a logical
+ * [num_pages, Hkv, 16, D] cache. Inside a block, token w and dim d sit at byte
+ *   (w / 8) * (D / 64) * 1024 + (d / 64) * 1024 + (w % 8) * 128
+ *     + (((d % 64) / 8) XOR (w % 8)) * 16 + (d % 8) * 2:
+ * 8-token groups of 128-byte rows with the 128-byte swizzle, so one
+ * contiguous copy per page lands in shared memory exactly as the tensor core
+ * reads it. A model writing its K/V can write this layout directly.
+ * pack: src logical -> dst TAPS layout; unpack: the reverse. src and dst are
+ * device buffers of num_pages * Hkv * 16 * D bf16, 16-byte aligned, distinct.
+ * ---------------------------------------------------------------------- */
+int taps_pack_kv_pages(const void* src, void* dst, int64_t num_pages, int Hkv, int D,
+                       void* stream);
+int taps_unpack_kv_pages(const void* src, void* dst, int64_t num_pages, int Hkv, int D,
+                         void* stream);
 
 /* ------------------------------------------------------------------------
  * taps_accept - lossless greedy acceptance (Sec. 4.1, Limitations): from the

@@ -6,6 +6,7 @@ taps_build_tree_mask, taps_tree_verify_attn and taps_accept. Importing the
 package fails when the library has not been built (no CPU fallback).
 """
 from ._binding import (LIB_PATH, TAPS_DEVFAULT_PAGE, TapsError, lib, scorer_params,  # noqa: F401
+                       taps_pack_kv_pages, taps_unpack_kv_pages,
                        taps_accept, taps_build_tree_mask, taps_score_reach, taps_select_subtree,
                        taps_topk_marginals, taps_tree_verify_attn,
                        topk_marginals_workspace_bytes, tree_verify_attn_workspace_bytes)

@@ -311,3 +311,38 @@ def taps_topk_marginals_noalloc(logits: torch.Tensor, K: int, out, stream=None):
                                          _stream(stream, logits.device))
     _check("taps_topk_marginals_noalloc", st)
     return ids, logp, lse, ent
+
+
+# ---------------------------------------------------------------------------
+# KV cache layout conversion
+# ---------------------------------------------------------------------------
+
+lib.taps_pack_kv_pages.argtypes = [_P, _P, _I64, _I, _I, _P]
+lib.taps_pack_kv_pages.restype = _I
+lib.taps_unpack_kv_pages.argtypes = [_P, _P, _I64, _I, _I, _P]
+lib.taps_unpack_kv_pages.restype = _I
+
+
+def taps_pack_kv_pages(cache: torch.Tensor, out: torch.Tensor | None = None, stream=None):
+    """Logical [num_pages, Hkv, 16, D] bf16 cache -> the TAPS page layout
+    (same shape and size; element order inside each (page, head) block)."""
+    _need(cache, torch.bfloat16, None, "cache")
+    num_pages, Hkv, P, D = cache.shape
+    if P != 16:
+        raise ValueError("pages hold 16 tokens")
+    out = torch.empty_like(cache) if out is None else out
+    st = lib.taps_pack_kv_pages(_ptr(cache), _ptr(out), num_pages, Hkv, D,
+                                _stream(stream, cache.device))
+    _check("taps_pack_kv_pages", st)
+    return out
+
+
+def taps_unpack_kv_pages(cache: torch.Tensor, out: torch.Tensor | None = None, stream=None):
+    """The TAPS page layout -> logical [num_pages, Hkv, 16, D]."""
+    _need(cache, torch.bfloat16, None, "cache")
+    num_pages, Hkv, P, D = cache.shape
+    out = torch.empty_like(cache) if out is None else out
+    st = lib.taps_unpack_kv_pages(_ptr(cache), _ptr(out), num_pages, Hkv, D,
+                                  _stream(stream, cache.device))
+    _check("taps_unpack_kv_pages", st)
+    return out

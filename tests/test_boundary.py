@@ -52,8 +52,8 @@ def test_workspace_queries_are_host_only(lib):
     tb = _b()
     assert tb.topk_marginals_workspace_bytes(1, 16, 151936, 8) > 0
     assert tb.topk_marginals_workspace_bytes(1, 16, 151936, 33) == 0      # K > 32
-    assert tb.tree_verify_attn_workspace_bytes(1, 64, 32, 8, 128, 4096) > 0
-    # enough independent work: no split, no workspace
+    # attention combines context chunks on chip: never a workspace
+    assert tb.tree_verify_attn_workspace_bytes(1, 64, 32, 8, 128, 4096) == 0
     assert tb.tree_verify_attn_workspace_bytes(32, 64, 32, 8, 128, 8192) == 0
 
 
@@ -115,5 +115,5 @@ def test_attention_rejects_bad_arguments(lib):
     assert call(D=96) == 2
     assert call(P=32) == 2
     assert call(Hq=80, Hkv=8) == 2                                   # group 10 > 8
-    assert call(ws=None) == 3                                        # split needs workspace
-    assert call(ws=FAKE, wsb=16) == 3
+    assert call(Hq=24, Hkv=8) == 2                                   # group 3
+    assert call(ctx=65536 - 63) == 2                                 # ctx + n_max > 65536

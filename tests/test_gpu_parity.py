@@ -268,6 +268,9 @@ def _attn_inputs(cfg, B, n_nodes, ctx, n_max, device_kv=False, seed=0):
 
 
 def _run_attn(taps, q, kc, vc, bt, ctx, n_nodes, mask, status=None):
+    """kc, vc: logical [num_pages, Hkv, 16, D] caches, packed here."""
+    kc = taps.taps_pack_kv_pages(kc)
+    vc = taps.taps_pack_kv_pages(vc)
     out, lse = taps.taps_tree_verify_attn(q, kc, vc, dt(bt), dt(ctx), dt(n_nodes),
                                           dt(mask.view(np.int32)), int(ctx.max()),
                                           want_lse=True, status=status)
@@ -358,6 +361,29 @@ def test_attention_bad_page_sets_status(taps):
     assert int(status.item()) == 0
 
 
+@pytest.mark.parametrize("D", [64, 128])
+def test_kv_pack_layout(taps, D):
+    """The packed cache puts token w, dim d of each (page, head) block at the
+    byte offset the header documents; unpack inverts pack."""
+    rng = np.random.default_rng(D)
+    num_pages, Hkv = 5, 3
+    x = rng.standard_normal((num_pages, Hkv, 16, D)).astype(np.float32)
+    xd = bf(x)
+    packed = taps.taps_pack_kv_pages(xd)
+    back = taps.taps_unpack_kv_pages(packed)
+    torch.cuda.synchronize()
+    assert torch.equal(back, xd)
+    raw = packed.view(torch.int16).cpu().numpy().reshape(num_pages * Hkv, -1)
+    src = xd.view(torch.int16).cpu().numpy().reshape(num_pages * Hkv, 16, D)
+    ch = D // 64
+    for blk in range(num_pages * Hkv):
+        for w in range(16):
+            for d in range(D):
+                off = ((w // 8) * ch * 1024 + (d // 64) * 1024 + (w % 8) * 128
+                       + ((((d % 64) // 8) ^ (w % 8)) * 16) + (d % 8) * 2)
+                assert raw[blk, off // 2] == src[blk, w, d]
+
+
 # ---------------------------------------------------------------------------
 # Stage 6
 # ---------------------------------------------------------------------------
@@ -446,7 +472,8 @@ def test_round_end_to_end(taps, name, n_max):
         kn, vn = W.make_kv_numpy(cfg, num_pages)
         qn = W.make_q_numpy(cfg, cfg.B, n_max)
         out = torch.empty((cfg.B, n_max, cfg.Hq, cfg.D), dtype=torch.bfloat16, device=DEV)
-        r.verify_layer(bf(qn), bf(kn), bf(vn), dt(bt), dt(ctx), out)
+        r.verify_layer(bf(qn), taps.taps_pack_kv_pages(bf(kn)), taps.taps_pack_kv_pages(bf(vn)),
+                       dt(bt), dt(ctx), out)
         torch.cuda.synchronize()
         rows = {(0, i, h) for i in range(0, int(sel["n_nodes"][0]), 7) for h in (0, cfg.Hq - 1)}
         o_ref, _ = O.tree_verify_attn(qn, kn, vn, bt, ctx, sel["n_nodes"], mask, only=rows)
