@@ -4,31 +4,38 @@
 //
 // Rows of one KV head are (node, query head of its GQA group) pairs, row
 // r = node * group + g, so every K/V tile is read once for the whole group.
-// One CTA owns up to 256 rows (two 128-row MMA tiles) of one KV head and one
-// chunk of the logical sequence [0, ctx_len + n_nodes). When there are fewer
-// (request, KV head, row block) units than SMs, the chunks of one unit form a
-// thread-block cluster: each CTA stages its normalised rows and (max, sum) in
-// shared memory and, after a cluster barrier, reduces a slice of the rows over
-// every CTA of the cluster through distributed shared memory, so no partial
-// result ever leaves the chip and no second kernel is needed.
+// One CTA owns 128 rows (one MMA tile) of one KV head and one chunk of the
+// logical sequence [0, ctx_len + n_nodes). When there are fewer (request, KV
+// head, row block) units than SMs, the chunks of one unit form a thread-block
+// cluster: each CTA stages its normalised rows and (max, sum) in shared
+// memory and, after a cluster barrier, reduces a slice of the rows over every
+// CTA of the cluster through distributed shared memory, so no partial result
+// ever leaves the chip and no second kernel is needed.
 //
-// Inside a CTA (10 warps):
-//   warp 0   TMA producer (one thread): Q rows once (4D box), then per 64-token
-//            tile one contiguous bulk copy per page for K and for V into a
-//            3-stage ring; the chunk's page ids are first copied to shared
-//            memory by the whole warp. The cache uses the TAPS page layout
-//            (see taps_pack_kv_pages): a (page, head) block is stored exactly
-//            as the tensor core reads it, 8-token groups of 128-byte swizzled
-//            rows, so one copy per page feeds the MMAs directly.
-//   warp 1   allocates 512 TMEM columns and issues every tcgen05.mma:
-//            S = Q K^T (M=128, N=64, K=D) into a double-buffered S region, then
-//            O += P V (M=128, N=D, K=64) into the O region.
-//   warps 2-9 softmax, one thread per row (TMEM lane): read S, apply the tree
-//            mask, online softmax in base 2 with lazy rescaling (O is rescaled
-//            in TMEM only when the running max grows by more than 2^8), write
-//            P as bf16 into shared memory for the PV MMA; finally normalise O
-//            and stage it (swizzled bf16) in the freed Q buffer, from where a
-//            TMA tensor store (one chunk) or the cluster reduction writes it.
+// Inside a CTA (8 warps):
+//   warps 0, 2  TMA producers (one thread each): warp 0 loads Q once (4D box)
+//            and the K tiles into a 3-stage ring, warp 2 the V tiles into a
+//            2-stage ring, one contiguous bulk copy per 16-token page of a
+//            128-token tile; the chunk's page ids are first copied to shared
+//            memory by the whole of warp 0. The cache uses the TAPS page
+//            layout (see taps_pack_kv_pages): a (page, head) block is stored
+//            exactly as the tensor core reads it, 8-token groups of 128-byte
+//            swizzled rows, so one copy per page feeds the MMAs directly.
+//   warp 1   allocates all 512 TMEM columns and issues every tcgen05.mma.
+//            S = Q K^T (M=128, N=128, K=D) goes to one of three S buffers;
+//            O += P V (M=128, N=D, K=16 per page) reads P from TMEM. After
+//            the softmax of tile j, one burst issues the PV of tile j and the
+//            QK of tile j+2 alternately, so consecutive MMAs never chain on
+//            one accumulator, while the softmax of tile j+1 already runs.
+//   warps 4-7 softmax, one thread per row (TMEM lane): read S, apply the
+//            tree mask, online softmax in base 2 with lazy rescaling (O is
+//            rescaled in TMEM only when the running max grows by more than
+//            2^8), and write P as bf16 over the S columns it came from;
+//            finally normalise O and stage it (swizzled bf16) in the freed Q
+//            buffer, from where a TMA tensor store (one chunk) or the cluster
+//            reduction writes it.
+// TMEM columns: O at [0, D), S (fp32) and then P (bf16 pairs) of buffer u at
+// [128 + 128 u, 256 + 128 u), u = 0, 1, 2; tile j uses buffer j mod 3.
 // Every wait is bounded; a wait that runs out sets TAPS_DEVFAULT_TIMEOUT and
 // the CTA winds down (waiting for its own copies and MMAs) before freeing TMEM.
 // Launches use programmatic dependent launch: a grid may start its set-up
@@ -45,16 +52,20 @@ namespace attn {
 
 using namespace sm100;
 
-constexpr int kRowsPerCta = 256;
-constexpr int kTile = 64;          // tokens per K/V tile (four 16-token pages)
-constexpr int kStages = 3;
-constexpr int kThreadsTc = 320;
+constexpr int kRowsPerCta = 128;
+constexpr int kTile = 128;             // tokens per K/V tile
+constexpr int kTilePages = kTile / 16;  // 16-token pages per tile
+constexpr int kKStages = 3;            // K tiles in flight (released after QK)
+constexpr int kVStages = 2;            // V tiles in flight (released after PV)
+constexpr int kSBufs = 3;              // S / P buffers in TMEM
+constexpr int kThreadsTc = 256;
 constexpr uint32_t kTmemCols = 512;
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 constexpr float kRescaleThreshold = 8.0f;
 constexpr int kMaxCluster = 16;
-constexpr int kMaxTokens = 65536;   // ctx_len + n_max per request (page ids kept in shared memory)
+constexpr int kMaxTokens = 65536;   // ctx_len + n_max per request
+constexpr int kMaxChunkTokens = 32768;   // page ids of one chunk are kept in shared memory
 
 struct Plan {
   int group, rows_max, m_blocks, cs, chunk_len;   // cs = chunks per unit = cluster size
@@ -69,12 +80,15 @@ inline Plan make_plan(int B, int n_max, int Hq, int Hkv, int max_ctx, const int*
   const int64_t units = static_cast<int64_t>(B) * Hkv * p.m_blocks;
   const int max_total = max_ctx + n_max;
   const int want = static_cast<int>(std::min<int64_t>(kMaxCluster, (kTargetSms + units - 1) / units));
-  const int cap = std::max(1, (max_total + 2 * kTile - 1) / (2 * kTile));
+  const int cap = std::max(1, (max_total + kTile - 1) / kTile);
   int cs = 1;
   for (int c = 2; c <= std::min(want, cap); ++c)
     if (max_active && units <= max_active[c]) cs = c;
+  cs = std::max(cs, (max_total + kMaxChunkTokens - 1) / kMaxChunkTokens);
   int chunk = (max_total + cs - 1) / cs;
-  chunk = (chunk + 15) / 16 * 16;                  // whole pages
+  // whole tiles where the chunk spans more than one, else whole pages: only
+  // the chunk holding the end of the sequence then ends inside a tile
+  chunk = chunk > kTile ? (chunk + kTile - 1) / kTile * kTile : (chunk + 15) / 16 * 16;
   p.chunk_len = chunk;
   p.cs = (max_total + chunk - 1) / chunk;
   return p;
@@ -105,28 +119,40 @@ struct Maps {
 template <int D>
 struct Smem {
   static constexpr int kChunks = D / 64;                      // 64-dim (128-byte) halves
-  static constexpr uint32_t kQ = 0;                           // [2 mt][chunks][128 rows][128 B]
-  static constexpr uint32_t kQBytes = 2 * kChunks * 16384;
-  static constexpr uint32_t kKV = kQBytes;                    // [stage][K 4 pages | V 4 pages], TAPS page layout
-  static constexpr uint32_t kKVStage = 2 * kChunks * 8192;
   static constexpr uint32_t kPageBytes = 16 * D * 2;          // one (page, head) block
   static constexpr uint32_t kGroupStride = kChunks * 1024;    // 8-token groups in a block
-  static constexpr uint32_t kP = kKV + kStages * kKVStage;    // [2 mt][128 rows][128 B]
-  static constexpr uint32_t kBar = kP + 2 * 16384;
-  static constexpr int kNumBars = 2 * kStages + 6;
-  static constexpr uint32_t kColMask = kBar + 8 * kNumBars;
-  static constexpr uint32_t kTmemSlot = kColMask + 8 * kStages;
+  static constexpr uint32_t kTileBytes = kTilePages * kPageBytes;   // one K or V tile
+  static constexpr uint32_t kQ = 0;                           // [chunks][128 rows][128 B]
+  static constexpr uint32_t kQBytes = kChunks * 16384;
+  static constexpr uint32_t kK = kQBytes;                     // K ring, TAPS page layout
+  static constexpr uint32_t kV = kK + kKStages * kTileBytes;  // V ring
+  static constexpr uint32_t kBar = kV + kVStages * kTileBytes;
+  static constexpr int kNumBars = 2 * kKStages + 2 * kVStages + 2 * kSBufs + 4;
+  static constexpr uint32_t kTmemSlot = kBar + 8 * kNumBars;
   static constexpr uint32_t kAbort = kTmemSlot + 4;
-  static constexpr uint32_t kMl = (kAbort + 4 + 7) / 8 * 8;   // [256] (max, sum) of the rows
+  static constexpr uint32_t kMl = (kAbort + 4 + 7) / 8 * 8;   // [128] (max, sum) of the rows
   static constexpr uint32_t kPages = kMl + 8 * kRowsPerCta;   // page ids of this CTA's chunk
-  static constexpr int kMaxChunkPages = kMaxTokens / 16;
+  static constexpr int kMaxChunkPages = kMaxChunkTokens / 16;
   static constexpr uint32_t kBytes = kPages + 4 * kMaxChunkPages;
-  static constexpr uint32_t kAlloc = kBytes + 1024;           // slack for the 1024-byte alignment
+  // at least half of the SM's shared memory, so that two CTAs (which would
+  // contend for the 512 TMEM columns) never share an SM
+  static constexpr uint32_t kAlloc = std::max<uint32_t>(kBytes + 1024, 120 * 1024);
 };
 
 __device__ __forceinline__ void set_fault(volatile int* abort_flag, int32_t* status, int bit) {
   *abort_flag = 1;
   if (status) atomicOr(status, bit);
+}
+
+// 64 columns of a row's ancestor mask starting at tree node jn0 (>= 0), from
+// the row's W 32-bit words; nodes past the last word are not visible.
+__device__ __forceinline__ uint64_t mask_window(const uint32_t* mrow, int W, int jn0) {
+  const int q = jn0 >> 5, o = jn0 & 31;
+  const uint32_t w0 = q < W ? mrow[q] : 0u;
+  const uint32_t w1 = q + 1 < W ? mrow[q + 1] : 0u;
+  const uint32_t w2 = q + 2 < W ? mrow[q + 2] : 0u;
+  const uint64_t lo = (static_cast<uint64_t>(w1) << 32) | w0;
+  return o == 0 ? lo : ((lo >> o) | (static_cast<uint64_t>(w2) << (64 - o)));
 }
 
 template <int D>
@@ -139,14 +165,19 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   const uint32_t sb = smem_u32(smem);
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + S::kBar);
-  uint64_t* kv_full = bars;
-  uint64_t* kv_empty = bars + kStages;
-  uint64_t* s_full = bars + 2 * kStages;
-  uint64_t* p_full = s_full + 2;
-  uint64_t* pv_done = p_full + 1;
-  uint64_t* q_full = pv_done + 1;
+  uint64_t* k_full = bars;
+  uint64_t* k_empty = k_full + kKStages;
+  uint64_t* v_full = k_empty + kKStages;
+  uint64_t* v_empty = v_full + kVStages;
+  uint64_t* s_full = v_empty + kVStages;   // [kSBufs] S of a tile written
+  // [kSBufs] P of a tile written (4 warps arrive). One per buffer: the
+  // softmax may finish tile j+1 before the MMA warp has waited for tile j,
+  // and a single barrier would then complete two phases in a row
+  uint64_t* p_full = s_full + kSBufs;
+  uint64_t* pv_done = p_full + kSBufs;     // the burst holding PV of a tile done
+  uint64_t* o_full = pv_done + 1;          // last PV done
+  uint64_t* q_full = o_full + 1;
   uint64_t* drain = q_full + 1;
-  uint64_t* colmask = reinterpret_cast<uint64_t*>(smem + S::kColMask);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + S::kTmemSlot);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + S::kAbort);
   const int warp = threadIdx.x >> 5;
@@ -170,13 +201,12 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
   const int total = C + n;
   const int rows = n * pl.group;
   const int row0 = mb * kRowsPerCta;
-  const int m_tiles = max(0, min(2, (rows - row0 + 127) / 128));
   const int pos0 = split * pl.chunk_len;
   const int pos1 = min(pos0 + pl.chunk_len, total);
   const int n_tiles = pos1 > pos0 ? (pos1 - pos0 + kTile - 1) / kTile : 0;
   const bool single = pl.cs == 1;
 
-  if (m_tiles == 0) {
+  if (row0 >= rows) {
     // no row of this block is live (the same for every CTA of a cluster): the
     // first chunk writes the block's padding rows as zeros
     if (split == 0) {
@@ -201,307 +231,340 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
   }
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kStages; ++s) {
-      mbar_init(&kv_full[s], 1);
-      mbar_init(&kv_empty[s], 1);
+    for (int s = 0; s < kKStages; ++s) {
+      mbar_init(&k_full[s], 1);
+      mbar_init(&k_empty[s], 1);
     }
-    mbar_init(&s_full[0], 1);
-    mbar_init(&s_full[1], 1);
-    mbar_init(p_full, 128 * m_tiles);
+    for (int s = 0; s < kVStages; ++s) {
+      mbar_init(&v_full[s], 1);
+      mbar_init(&v_empty[s], 1);
+    }
+    for (int u = 0; u < kSBufs; ++u) {
+      mbar_init(&s_full[u], 1);
+      mbar_init(&p_full[u], 4);
+    }
     mbar_init(pv_done, 1);
+    mbar_init(o_full, 1);
     mbar_init(q_full, 1);
     mbar_init(drain, 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  const uint32_t tmem = *tmem_slot;
-  // TMEM columns: O of M-tile mt at mt * D; S of buffer u, M-tile mt at 256 + u*128 + mt*64
-  auto o_col = [](int mt) { return static_cast<uint32_t>(mt * D); };
-  auto s_col = [](int u, int mt) { return static_cast<uint32_t>(256 + u * 128 + mt * 64); };
-
-  if (n_tiles == 0) {
-    // this chunk is empty for this request: nothing to compute, the epilogue
-    // below contributes zero rows with an empty softmax
-  } else if (warp == 0) {
-    // ------------------------------------------------------------ TMA producer
-    // page ids of the whole chunk -> shared memory (whole warp, coalesced);
-    // -1 marks a logical page missing from the block table
-    int32_t* spages = reinterpret_cast<int32_t*>(smem + S::kPages);
+  // page ids of the whole chunk -> shared memory (producer warp, coalesced);
+  // -1 marks a logical page missing from the block table
+  int32_t* spages = reinterpret_cast<int32_t*>(smem + S::kPages);
+  if (warp == 0) {
     const int32_t* bt = a.block_table + static_cast<int64_t>(b) * a.max_pages;
     const int lp0 = pos0 >> 4;
     const int npg = (pos1 - pos0 + 15) >> 4;
     for (int i = lane; i < npg; i += 32) spages[i] = lp0 + i < a.max_pages ? bt[lp0 + i] : -1;
-    __syncwarp();
-    if (lane == 0) {
-      const uint64_t policy = l2_evict_first_policy();
-      int issued = 0;
-      for (int j = 0; j < n_tiles; ++j) {
-        if (*abort_flag) break;
-        const int s = j % kStages;
-        if (j >= kStages && !mbar_wait(&kv_empty[s], ((j / kStages) - 1) & 1)) {
-          set_fault(abort_flag, a.status, TAPS_DEVFAULT_TIMEOUT);
-          break;
-        }
-        const int t0 = pos0 + j * kTile;
-        int pages[4];
-        uint64_t cm = 0;
-        uint32_t bytes = 0;
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  // validity of the 64 columns [64 h, 64 h + 64) of tile j: inside the chunk
+  // and on a valid page, 16 bits per page
+  auto tile_cols = [&](int j, int h) -> uint64_t {
+    const int t0 = pos0 + j * kTile + 64 * h;
+    uint64_t cm = 0;
 #pragma unroll
-        for (int p = 0; p < 4; ++p) {
-          pages[p] = -1;
-          const int tp = t0 + 16 * p;
-          if (tp >= pos1) continue;
-          const int pg = spages[j * 4 + p];
-          if (pg < 0 || pg >= a.num_pages) {
-            if (a.status) atomicOr(a.status, TAPS_DEVFAULT_PAGE);
-            continue;
-          }
-          pages[p] = pg;
-          bytes += 2 * CH * 2048;
-          const int nv = min(16, pos1 - tp);
-          cm |= (nv == 16 ? 0xFFFFull : ((1ull << nv) - 1)) << (16 * p);
-        }
-        colmask[s] = cm;
-        mbar_arrive_expect_tx(&kv_full[s], bytes);
-        const uint32_t kbase = sb + S::kKV + s * S::kKVStage;
-#pragma unroll
-        for (int p = 0; p < 4; ++p) {
-          if (pages[p] < 0) continue;
-          const int64_t blk = (static_cast<int64_t>(pages[p]) * a.Hkv + kv) * (16 * D);
-          bulk_load(kbase + p * S::kPageBytes, a.k + blk, S::kPageBytes, &kv_full[s], policy);
-          bulk_load(kbase + 4 * S::kPageBytes + p * S::kPageBytes, a.v + blk, S::kPageBytes,
-                    &kv_full[s], policy);
-        }
-        if (j == 0) {
-          // Q rows of this block (issued after the first K/V tile, which comes
-          // from DRAM): one box of (64 dims, group heads, 128/group nodes) per
-          // M-tile and 64-dim half; nodes past n_max read as zeros
-          mbar_arrive_expect_tx(q_full, static_cast<uint32_t>(m_tiles * CH * 16384));
-          for (int mt = 0; mt < m_tiles; ++mt)
-            for (int c = 0; c < CH; ++c)
-              tma_load_4d(sb + S::kQ + (mt * CH + c) * 16384, &maps.q, q_full, c * 64,
-                          kv * pl.group, (row0 + mt * 128) / pl.group, b);
-        }
-        issued = j + 1;
+    for (int p = 0; p < 4; ++p) {
+      const int tp = t0 + 16 * p;
+      if (tp >= pos1) continue;
+      const int pg = spages[j * kTilePages + 4 * h + p];
+      if (pg < 0 || pg >= a.num_pages) continue;
+      const int nv = min(16, pos1 - tp);
+      cm |= (nv == 16 ? 0xFFFFull : ((1ull << nv) - 1)) << (16 * p);
+    }
+    return cm;
+  };
+  constexpr uint32_t kOCol = 0;
+  auto s_col = [](int u) { return static_cast<uint32_t>(128 + u * 128); };
+
+  if (n_tiles == 0) {
+    // this chunk is empty for this request: nothing to compute, the epilogue
+    // below contributes zero rows with an empty softmax
+  } else if (warp == 0 || warp == 2) {
+    // ------------------------------------------------------------ TMA producers
+    // warp 0 streams Q and the K tiles, warp 2 the V tiles, each into its own
+    // ring, so neither producer's wait stalls the other. Lane p handles page
+    // p of a tile: its page id is fetched one tile ahead, and the eight bulk
+    // copies of a tile leave in one warp instruction.
+    const bool is_k = warp == 0;
+    const int nst = is_k ? kKStages : kVStages;
+    uint64_t* full = is_k ? k_full : v_full;
+    uint64_t* empty = is_k ? k_empty : v_empty;
+    const __nv_bfloat16* cache = is_k ? a.k : a.v;
+    const uint32_t ring = sb + (is_k ? S::kK : S::kV);
+    const uint64_t policy = l2_evict_first_policy();
+    if (is_k && lane == 0) {
+      // Q rows of this block first: one box of (64 dims, group heads,
+      // 128/group nodes) per 64-dim half; nodes past n_max read as zeros
+      mbar_arrive_expect_tx(q_full, static_cast<uint32_t>(CH * 16384));
+      for (int c = 0; c < CH; ++c)
+        tma_load_4d(sb + S::kQ + c * 16384, &maps.q, q_full, c * 64, kv * pl.group,
+                    row0 / pl.group, b);
+    }
+    auto in_chunk = [&](int j) { return lane < kTilePages && pos0 + j * kTile + 16 * lane < pos1; };
+    int pg = in_chunk(0) ? spages[lane] : -1;
+    int issued = 0;
+    for (int j = 0; j < n_tiles; ++j) {
+      if (__any_sync(kFullMask, *abort_flag != 0)) break;
+      const int s = j % nst;
+      if (j >= nst && !__all_sync(kFullMask, mbar_wait(&empty[s], ((j / nst) - 1) & 1))) {
+        if (lane == 0) set_fault(abort_flag, a.status, TAPS_DEVFAULT_TIMEOUT);
+        break;
       }
-      // never leave the CTA with copies in flight
-      if (issued > 0) mbar_wait(q_full, 0);
-      for (int j = max(0, issued - kStages); j < issued; ++j)
-        mbar_wait(&kv_full[j % kStages], (j / kStages) & 1);
+      const bool valid = pg >= 0 && pg < a.num_pages;
+      if (is_k && in_chunk(j) && !valid && a.status) atomicOr(a.status, TAPS_DEVFAULT_PAGE);
+      const uint32_t vm = __ballot_sync(kFullMask, valid);
+      if (lane == 0) mbar_arrive_expect_tx(&full[s], __popc(vm) * S::kPageBytes);
+      __syncwarp();
+      if (valid) {
+        const int64_t blk = (static_cast<int64_t>(pg) * a.Hkv + kv) * (16 * D);
+        bulk_load(ring + s * S::kTileBytes + lane * S::kPageBytes, cache + blk, S::kPageBytes,
+                  &full[s], policy);
+      }
+      issued = j + 1;
+      if (j + 1 < n_tiles) pg = in_chunk(j + 1) ? spages[(j + 1) * kTilePages + lane] : -1;
+    }
+    // never leave the CTA with copies in flight
+    if (lane == 0) {
+      if (is_k) mbar_wait(q_full, 0);
+      for (int j = max(0, issued - nst); j < issued; ++j) mbar_wait(&full[j % nst], (j / nst) & 1);
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
     constexpr uint32_t idesc_qk = idesc_bf16_f32(128, kTile, false, false);
     constexpr uint32_t idesc_pv = idesc_bf16_f32(128, D, false, true);
+    constexpr int kQkSteps = D / 16;
+    auto qk_step = [&](int jj, int ks) {
+      const uint32_t kb = sb + S::kK + (jj % kKStages) * S::kTileBytes;
+      const uint64_t ad = sw128_desc(sb + S::kQ + (ks / 4) * 16384 + (ks % 4) * 32, 16, 1024);
+      const uint64_t bd = sw128_desc(kb + (ks / 4) * 1024 + (ks % 4) * 32, 16, S::kGroupStride);
+      mma_bf16(tmem + s_col(jj % kSBufs), ad, bd, idesc_qk, ks > 0 ? 1u : 0u);
+    };
     bool ok = __all_sync(kFullMask, mbar_wait(q_full, 0));
-    if (!ok && lane == 0) set_fault(abort_flag, a.status, TAPS_DEVFAULT_TIMEOUT);
-    for (int j = 0; ok && j <= n_tiles; ++j) {
-      if (__any_sync(kFullMask, *abort_flag != 0)) break;
-      if (j < n_tiles) {
-        const int s = j % kStages;
-        if (!__all_sync(kFullMask, mbar_wait(&kv_full[s], (j / kStages) & 1))) {
-          if (lane == 0) set_fault(abort_flag, a.status, TAPS_DEVFAULT_TIMEOUT);
-          break;
-        }
-        const uint64_t cm = colmask[s];
-        if (cm != ~0ull) {
-          // rows of skipped or out-of-chunk positions: zero V so that P = 0
-          // never meets stale (possibly non-finite) data
-          uint8_t* vb = smem + S::kKV + s * S::kKVStage + 4 * S::kPageBytes;
-          for (int e = lane; e < kTile * 8 * CH; e += 32) {
-            const int t = e / (8 * CH), c = (e / 8) % CH, q16 = e % 8;
-            const int p = t >> 4, w = t & 15;
-            if (!((cm >> t) & 1ull))
-              *reinterpret_cast<uint4*>(vb + p * S::kPageBytes + (w >> 3) * S::kGroupStride +
-                                        c * 1024 + (w & 7) * 128 + q16 * 16) = make_uint4(0, 0, 0, 0);
-          }
-          fence_proxy_async_smem();
-        }
-        __syncwarp();
-        if (lane == 0) {
-          tc_fence_after();
-          const uint32_t kb = sb + S::kKV + s * S::kKVStage;
-          for (int mt = 0; mt < m_tiles; ++mt) {
+    // QK of the first two tiles
+    for (int jj = 0; ok && jj < min(2, n_tiles); ++jj) {
+      ok = __all_sync(kFullMask, mbar_wait(&k_full[jj % kKStages], (jj / kKStages) & 1));
+      if (ok && lane == 0) {
+        tc_fence_after();
 #pragma unroll
-            for (int ks = 0; ks < D / 16; ++ks) {
-              const uint64_t ad =
-                  sw128_desc(sb + S::kQ + (mt * CH + ks / 4) * 16384 + (ks % 4) * 32, 16, 1024);
-              const uint64_t bd =
-                  sw128_desc(kb + (ks / 4) * 1024 + (ks % 4) * 32, 16, S::kGroupStride);
-              mma_bf16(tmem + s_col(j & 1, mt), ad, bd, idesc_qk, ks > 0 ? 1u : 0u);
-            }
-          }
-          mma_commit(&s_full[j & 1]);
-        }
-        __syncwarp();
+        for (int ks = 0; ks < kQkSteps; ++ks) qk_step(jj, ks);
+        mma_commit(&s_full[jj % kSBufs]);
+        mma_commit(&k_empty[jj % kKStages]);
       }
-      if (j >= 1) {
-        const int jp = j - 1, sp = jp % kStages;
-        if (!__all_sync(kFullMask, mbar_wait(p_full, jp & 1))) {
-          if (lane == 0) set_fault(abort_flag, a.status, TAPS_DEVFAULT_TIMEOUT);
-          break;
-        }
-        if (lane == 0) {
-          tc_fence_after();
-          const uint32_t vb = sb + S::kKV + sp * S::kKVStage + 4 * S::kPageBytes;
-          for (int mt = 0; mt < m_tiles; ++mt) {
-#pragma unroll
-            for (int ks = 0; ks < kTile / 16; ++ks) {
-              const uint64_t ad = sw128_desc(sb + S::kP + mt * 16384 + ks * 32, 16, 1024);
-              const uint64_t bd = sw128_desc(vb + ks * S::kPageBytes, 1024, S::kGroupStride);
-              mma_bf16(tmem + o_col(mt), ad, bd, idesc_pv, (jp > 0 || ks > 0) ? 1u : 0u);
-            }
-          }
-          mma_commit(pv_done);
-          mma_commit(&kv_empty[sp]);
-        }
-        __syncwarp();
-      }
+      __syncwarp();
     }
+    bool o_started = false;   // O holds a first product
+    auto page_id = [&](int j) {
+      return lane < kTilePages && pos0 + j * kTile + 16 * lane < pos1
+                 ? spages[j * kTilePages + lane] : -1;
+    };
+    int pgv = page_id(0);
+    // burst j: PV of tile j (after its softmax) alternating with QK of tile j+2
+    for (int j = 0; ok && j < n_tiles; ++j) {
+      if (__any_sync(kFullMask, *abort_flag != 0)) break;
+      const int jn = j + 2;
+      const bool has_qk = jn < n_tiles;
+      const int sv = j % kVStages;
+      if (!__all_sync(kFullMask, mbar_wait(&v_full[sv], (j / kVStages) & 1))) {
+        ok = false;
+        break;
+      }
+      // pages of tile j holding a valid token (lane p: page p, id fetched
+      // during the previous burst), and the page cut by the end of the
+      // sequence, whose rows past the end are zeroed so that P = 0 never
+      // meets stale (possibly non-finite) data
+      const int tp = pos0 + j * kTile + 16 * lane;
+      const bool live = pgv >= 0 && pgv < a.num_pages;
+      const uint32_t page_live = __ballot_sync(kFullMask, live);
+      const uint32_t cut = __ballot_sync(kFullMask, live && pos1 - tp < 16);
+      if (cut) {
+        const int p = __ffs(cut) - 1;
+        const int nv = __shfl_sync(kFullMask, pos1 - tp, p);
+        uint8_t* pb = smem + S::kV + sv * S::kTileBytes + p * S::kPageBytes;
+        for (int e = lane; e < 16 * 8 * CH; e += 32) {
+          const int w = e / (8 * CH), c = (e / 8) % CH, q16 = e % 8;
+          if (w >= nv)
+            *reinterpret_cast<uint4*>(pb + (w >> 3) * S::kGroupStride + c * 1024 +
+                                      (w & 7) * 128 + q16 * 16) = make_uint4(0, 0, 0, 0);
+        }
+        fence_proxy_async_smem();
+      }
+      __syncwarp();
+      if (has_qk &&
+          !__all_sync(kFullMask, mbar_wait(&k_full[jn % kKStages], (jn / kKStages) & 1))) {
+        ok = false;
+        break;
+      }
+      if (!__all_sync(kFullMask, mbar_wait(&p_full[j % kSBufs], (j / kSBufs) & 1))) {
+        ok = false;
+        break;
+      }
+      if (lane == 0) {
+        tc_fence_after();
+        const uint32_t vb = sb + S::kV + sv * S::kTileBytes;
+        const uint32_t pcol = tmem + s_col(j % kSBufs);
+#pragma unroll
+        for (int ks = 0; ks < kTilePages; ++ks) {
+          if ((page_live >> ks) & 1u) {
+            const uint64_t bd = sw128_desc(vb + ks * S::kPageBytes, 1024, S::kGroupStride);
+            mma_bf16_ts(tmem + kOCol, pcol + ks * 8, bd, idesc_pv, o_started ? 1u : 0u);
+            o_started = true;
+          }
+          if (has_qk && ks < kQkSteps) qk_step(jn, ks);
+        }
+        mma_commit(pv_done);
+        mma_commit(&v_empty[sv]);
+        if (has_qk) {
+          mma_commit(&s_full[jn % kSBufs]);
+          mma_commit(&k_empty[jn % kKStages]);
+        }
+        if (j == n_tiles - 1) mma_commit(o_full);
+      }
+      __syncwarp();
+      if (j + 1 < n_tiles) pgv = page_id(j + 1);
+    }
+    if (!ok && lane == 0) set_fault(abort_flag, a.status, TAPS_DEVFAULT_TIMEOUT);
     // every MMA issued by this warp completes before TMEM is released
     if (lane == 0) mma_commit(drain);
     __syncwarp();
     mbar_wait(drain, 0);
   }
-  if (warp >= 2) {
+  if (warp >= 4) {
     // ------------------------------------------------------------ softmax warps
-    const int sw = warp - 2;
-    const int mt = sw >> 2;
+    // (also for an empty chunk: its epilogue stages zero rows for the peers)
     const int quarter = warp & 3;                  // TMEM lanes 32*quarter .. +31
-    const int r = quarter * 32 + lane;             // row within the M-tile
-    const int grow = row0 + mt * 128 + r;
-    const bool live = mt < m_tiles;
-    const bool valid_row = live && grow < rows;
+    const int r = quarter * 32 + lane;             // row of the block
+    const int grow = row0 + r;
+    const bool valid_row = grow < rows;
     const int node = valid_row ? grow / pl.group : 0;
     const uint32_t lane_base = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
     const float scale = a.scale_log2;
+    const uint32_t* mrow = a.mask + (static_cast<int64_t>(b) * a.n_max + node) * a.W;
     float m_used = -INFINITY, l = 0.f;
     bool ok = true;
-    const bool has_o = live && n_tiles > 0;
-    if (has_o) {
-      const uint32_t* mrow = a.mask + (static_cast<int64_t>(b) * a.n_max + node) * a.W;
-      uint8_t* prow = smem + S::kP + mt * 16384 + r * 128;
-      for (int j = 0; j < n_tiles; ++j) {
-        if (__any_sync(kFullMask, *abort_flag != 0)) { ok = false; break; }
-        const int s = j % kStages;
-        // kv_full of this tile completed before its QK MMA: this wait returns at
-        // once and makes the producer's column mask visible
-        if (!__all_sync(kFullMask, mbar_wait(&s_full[j & 1], (j >> 1) & 1) &&
-                                        mbar_wait(&kv_full[s], (j / kStages) & 1))) {
-          if (lane == 0) set_fault(abort_flag, a.status, TAPS_DEVFAULT_TIMEOUT);
-          ok = false;
-          break;
-        }
-        const uint64_t cm = colmask[s];
-        tc_fence_after();
-        uint32_t sv[64];
-        tmem_ld64_sync(lane_base + s_col(j & 1, mt), sv);
+    for (int j = 0; j < n_tiles; ++j) {
+      if (__any_sync(kFullMask, *abort_flag != 0)) { ok = false; break; }
+      // visible columns of this row in tile j, before waiting for S: these
+      // loads would queue behind the tensor core's shared-memory reads
+      uint64_t vis[2] = {0ull, 0ull};
+      if (valid_row) {
         const int t0 = pos0 + j * kTile;
-        uint64_t vis = valid_row ? cm : 0ull;
-        if (valid_row && t0 + kTile > C) {
-          // columns from i0 on are tree nodes jn = t0 + i - C: take a 64-bit
-          // window of this row's ancestor mask starting at node jn0
-          const int i0 = max(0, C - t0);
-          const int jn0 = t0 + i0 - C;
-          const int q = jn0 >> 5, o = jn0 & 31;
-          const uint32_t w0 = q < a.W ? mrow[q] : 0u;
-          const uint32_t w1 = q + 1 < a.W ? mrow[q + 1] : 0u;
-          const uint32_t w2 = q + 2 < a.W ? mrow[q + 2] : 0u;
-          const uint64_t lo = (static_cast<uint64_t>(w1) << 32) | w0;
-          const uint64_t win = o == 0 ? lo : ((lo >> o) | (static_cast<uint64_t>(w2) << (64 - o)));
-          const uint64_t ctx_cols = i0 == 0 ? 0ull : ((1ull << i0) - 1);
-          vis &= ctx_cols | (win << i0);
-        }
-        if (vis != ~0ull) {
 #pragma unroll
-          for (int i = 0; i < 64; ++i)
-            if (!((vis >> i) & 1ull)) sv[i] = 0xFF800000u;   // -inf
-        }
-        float mx[8];
-#pragma unroll
-        for (int k = 0; k < 8; ++k) mx[k] = __uint_as_float(sv[k]);
-#pragma unroll
-        for (int i = 8; i < 64; ++i) mx[i & 7] = fmaxf(mx[i & 7], __uint_as_float(sv[i]));
-        const float tmax =
-            fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
-                  fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7]))) * scale;
-        const float m_new = fmaxf(m_used, tmax);
-        const bool grow_max =
-            (m_used == -INFINITY) ? (m_new > -INFINITY) : (m_new > m_used + kRescaleThreshold);
-        float alpha = 1.f;
-        if (grow_max) {
-          alpha = (m_used == -INFINITY) ? 0.f : ex2_approx(m_used - m_new);
-          m_used = m_new;
-        }
-        uint32_t pk[32];
-        float acc[8];
-#pragma unroll
-        for (int k = 0; k < 8; ++k) acc[k] = 0.f;
-        if (m_used != -INFINITY) {
-          const float nm = -m_used;
-#pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            const float p0 = ex2_approx(fmaf(__uint_as_float(sv[2 * i]), scale, nm));
-            const float p1 = ex2_approx(fmaf(__uint_as_float(sv[2 * i + 1]), scale, nm));
-            pk[i] = pack_bf16x2(p0, p1);
-            acc[i & 7] += p0 + p1;
+        for (int h = 0; h < 2; ++h) {
+          vis[h] = tile_cols(j, h);
+          const int th = t0 + 64 * h;
+          if (th + 64 > C) {
+            // columns from i0 on are tree nodes jn = th + i - C
+            const int i0 = max(0, C - th);
+            const uint64_t win = mask_window(mrow, a.W, th + i0 - C);
+            const uint64_t ctx_cols = i0 == 0 ? 0ull : ((1ull << i0) - 1);
+            vis[h] &= ctx_cols | (win << i0);
           }
-        } else {
-#pragma unroll
-          for (int i = 0; i < 32; ++i) pk[i] = 0u;
         }
-        const float psum = ((acc[0] + acc[1]) + (acc[2] + acc[3])) +
-                           ((acc[4] + acc[5]) + (acc[6] + acc[7]));
-        l = l * alpha + psum;
-        // PV of the previous tile must be done before P is overwritten and O touched
-        if (j > 0 && !__all_sync(kFullMask, mbar_wait(pv_done, (j - 1) & 1))) {
-          if (lane == 0) set_fault(abort_flag, a.status, TAPS_DEVFAULT_TIMEOUT);
-          ok = false;
-          break;
-        }
-        const bool need_rescale = grow_max && j > 0 && alpha != 1.f;
-        if (__any_sync(kFullMask, need_rescale)) {
-          tc_fence_after();
-          const float f = need_rescale ? alpha : 1.f;
-#pragma unroll 1
-          for (int c = 0; c < D / 32; ++c) {
-            uint32_t o[32];
-            tmem_ld32_sync(lane_base + o_col(mt) + c * 32, o);
-#pragma unroll
-            for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * f);
-            tmem_st32(lane_base + o_col(mt) + c * 32, o);
-          }
-          tmem_wait_st();
-        }
-#pragma unroll
-        for (int j8 = 0; j8 < 8; ++j8)
-          *reinterpret_cast<uint4*>(prow + ((j8 ^ (r & 7)) << 4)) =
-              make_uint4(pk[4 * j8], pk[4 * j8 + 1], pk[4 * j8 + 2], pk[4 * j8 + 3]);
-        fence_proxy_async_smem();
-        tc_fence_before();
-        mbar_arrive(p_full);
       }
-      if (ok && !__all_sync(kFullMask, mbar_wait(pv_done, (n_tiles - 1) & 1))) {
+      const int u = j % kSBufs;
+      if (!__all_sync(kFullMask, mbar_wait(&s_full[u], (j / kSBufs) & 1))) {
         if (lane == 0) set_fault(abort_flag, a.status, TAPS_DEVFAULT_TIMEOUT);
         ok = false;
+        break;
       }
+      tc_fence_after();
+      uint32_t sv[128];
+      tmem_ld128_sync(lane_base + s_col(u), sv);
+      if ((vis[0] & vis[1]) != ~0ull) {
+#pragma unroll
+        for (int i = 0; i < 128; ++i)
+          if (!((vis[i >> 6] >> (i & 63)) & 1ull)) sv[i] = 0xFF800000u;   // -inf
+      }
+      float mx[8];
+#pragma unroll
+      for (int k = 0; k < 8; ++k) mx[k] = __uint_as_float(sv[k]);
+#pragma unroll
+      for (int i = 8; i < 128; ++i) mx[i & 7] = fmaxf(mx[i & 7], __uint_as_float(sv[i]));
+      const float tmax =
+          fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
+                fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7]))) * scale;
+      const float m_new = fmaxf(m_used, tmax);
+      const bool grow_max =
+          (m_used == -INFINITY) ? (m_new > -INFINITY) : (m_new > m_used + kRescaleThreshold);
+      float alpha = 1.f;
+      if (grow_max) {
+        alpha = (m_used == -INFINITY) ? 0.f : ex2_approx(m_used - m_new);
+        m_used = m_new;
+      }
+      float acc[8];
+#pragma unroll
+      for (int k = 0; k < 8; ++k) acc[k] = 0.f;
+      // P over the first 64 columns of this S buffer (the row's S is in
+      // registers), in two halves of 32 columns
+      const float nm = m_used == -INFINITY ? 0.f : -m_used;
+      const bool any = m_used != -INFINITY;
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        uint32_t pk[32];
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          const float p0 = any ? ex2_approx(fmaf(__uint_as_float(sv[64 * h + 2 * i]), scale, nm)) : 0.f;
+          const float p1 = any ? ex2_approx(fmaf(__uint_as_float(sv[64 * h + 2 * i + 1]), scale, nm)) : 0.f;
+          pk[i] = pack_bf16x2(p0, p1);
+          acc[i & 7] += p0 + p1;
+        }
+        tmem_st32(lane_base + s_col(u) + 32 * h, pk);
+      }
+      const float psum = ((acc[0] + acc[1]) + (acc[2] + acc[3])) +
+                         ((acc[4] + acc[5]) + (acc[6] + acc[7]));
+      l = l * alpha + psum;
+      // a grown max rescales O before P of this tile is released; the PV of
+      // the previous tile may still be running, so wait for it first
+      const bool need_rescale = grow_max && j > 0 && alpha != 1.f;
+      if (__any_sync(kFullMask, need_rescale)) {
+        if (!__all_sync(kFullMask, mbar_wait(pv_done, (j - 1) & 1))) {
+          if (lane == 0) set_fault(abort_flag, a.status, TAPS_DEVFAULT_TIMEOUT);
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const float f = need_rescale ? alpha : 1.f;
+#pragma unroll 1
+        for (int c = 0; c < D / 32; ++c) {
+          uint32_t o[32];
+          tmem_ld32_sync(lane_base + kOCol + c * 32, o);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * f);
+          tmem_st32(lane_base + kOCol + c * 32, o);
+        }
+      }
+      tmem_wait_st();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&p_full[u]);
     }
-    if (threadIdx.x == 64) pdl_launch_dependents();
-    // ---- epilogue. Once a live warp's last PV is done every MMA has finished,
-    // so the Q buffer is free: stage the normalised bf16 rows there in the
-    // same swizzled layout, and this row's (max, sum) next to them.
+    if (ok && n_tiles > 0 && !__all_sync(kFullMask, mbar_wait(o_full, 0))) {
+      if (lane == 0) set_fault(abort_flag, a.status, TAPS_DEVFAULT_TIMEOUT);
+      ok = false;
+    }
+    if (threadIdx.x == 128) pdl_launch_dependents();
+    // ---- epilogue. Once the last PV is done every MMA reading Q has
+    // finished: stage the normalised bf16 rows there in the same swizzled
+    // layout, and this row's (max, sum) next to them.
     const bool good = ok && valid_row && l > 0.f;
     const float inv = good ? 1.f / l : 0.f;
-    uint8_t* srow = smem + S::kQ + (mt * CH) * 16384 + r * 128;
-    if (has_o) {
+    uint8_t* srow = smem + S::kQ + r * 128;
+    if (n_tiles > 0 && __any_sync(kFullMask, good)) {
       tc_fence_after();
 #pragma unroll 1
       for (int c = 0; c < D / 64; ++c) {
         uint32_t o[64];
-        tmem_ld64_sync(lane_base + o_col(mt) + c * 64, o);
+        tmem_ld64_sync(lane_base + kOCol + c * 64, o);
+        if (!good) {
+#pragma unroll
+          for (int k = 0; k < 64; ++k) o[k] = 0u;
+        }
 #pragma unroll
         for (int k = 0; k < 8; ++k) {
           const int j16 = c * 8 + k;                      // 16-byte chunk of the row
@@ -519,7 +582,7 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
         *reinterpret_cast<uint4*>(srow + (j16 >> 3) * 16384 + (((j16 & 7) ^ (r & 7)) << 4)) =
             make_uint4(0, 0, 0, 0);
     }
-    reinterpret_cast<float2*>(smem + S::kMl)[mt * 128 + r] =
+    reinterpret_cast<float2*>(smem + S::kMl)[r] =
         good ? make_float2(m_used, l) : make_float2(-INFINITY, 0.f);
     if (single) {
       if (a.lse && grow < pl.rows_max) {
@@ -528,14 +591,11 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
         a.lse[orow] = good ? (m_used + log2f(l)) * kLn2 : 0.f;
       }
       fence_proxy_async_smem();
-      named_bar_sync(1, 256);
-      if (threadIdx.x == 64) {
-        for (int t = 0; t < 2; ++t) {
-          if (row0 + t * 128 >= pl.rows_max) break;
-          for (int c = 0; c < CH; ++c)
-            tma_store_4d(&maps.out, sb + S::kQ + (t * CH + c) * 16384, c * 64, kv * pl.group,
-                         (row0 + t * 128) / pl.group, b);
-        }
+      named_bar_sync(1, 128);
+      if (threadIdx.x == 128) {
+        for (int c = 0; c < CH; ++c)
+          tma_store_4d(&maps.out, sb + S::kQ + c * 16384, c * 64, kv * pl.group, row0 / pl.group,
+                       b);
         bulk_commit();
         bulk_wait_read_all();
       }
@@ -560,81 +620,86 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
   }
-  if (warp >= 2) {
-    constexpr int DPL = D / 32;                        // dims per lane
+  {
+    // a row is read by CPR lanes, 16 bytes each, so one warp instruction
+    // covers RPI rows; (max, sum) reductions stay inside each row's lanes
+    constexpr int CPR = D / 8;
+    constexpr int RPI = 32 / CPR;
+    constexpr int MLQ = (kMaxCluster + CPR - 1) / CPR;
+    constexpr int kWarps = kThreadsTc / 32;
     const int cs = pl.cs;
     const uint32_t rank = cluster_ctarank();
     const int per = (kRowsPerCta + cs - 1) / cs;
     const int rb = static_cast<int>(rank) * per;
     const int re = min(kRowsPerCta, rb + per);
-    const int boff = lane * DPL * 2;                   // this lane's bytes of a row
-    const int j16 = boff >> 4;
-    for (int rr = rb + (warp - 2); rr < re; rr += 8) {
+    const int sr = lane / CPR, q16 = lane % CPR;
+    const int seg0 = sr * CPR;
+    for (int base = rb + warp * RPI; base < re; base += kWarps * RPI) {
+      const int rr = base + sr;
       const int gr = row0 + rr;
-      if (gr >= pl.rows_max) break;
-      float2 mlv = make_float2(-INFINITY, 0.f);
-      if (lane < cs) {
-        const uint2 t = ld_cluster_v2(mapa_shared(sb + S::kMl + rr * 8, lane));
-        mlv = make_float2(__uint_as_float(t.x), __uint_as_float(t.y));
+      const bool valid = rr < re && gr < pl.rows_max;
+      // every remote load of the batch is issued before any is used
+      uint2 mlr[MLQ];
+      uint4 v[kMaxCluster];
+#pragma unroll
+      for (int m = 0; m < MLQ; ++m) {
+        const int q = q16 + m * CPR;
+        mlr[m] = (valid && q < cs) ? ld_cluster_v2(mapa_shared(sb + S::kMl + rr * 8, q))
+                                   : make_uint2(__float_as_uint(-INFINITY), 0u);
       }
-      float M = mlv.x;
+      const uint32_t laddr =
+          sb + S::kQ + (q16 >> 3) * 16384 + rr * 128 + (((q16 & 7) ^ (rr & 7)) << 4);
 #pragma unroll
-      for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(kFullMask, M, off));
-      const float w = mlv.y > 0.f ? mlv.y * ex2_approx(mlv.x - M) : 0.f;
-      float Lsum = w;
+      for (int q = 0; q < kMaxCluster; ++q)
+        v[q] = (valid && q < cs) ? ld_cluster_v4(mapa_shared(laddr, q)) : make_uint4(0, 0, 0, 0);
+      float M = -INFINITY;
 #pragma unroll
-      for (int off = 16; off > 0; off >>= 1) Lsum += __shfl_xor_sync(kFullMask, Lsum, off);
-      const int rmt = rr >> 7, rrow = rr & 127;
-      const uint32_t laddr = sb + S::kQ + (rmt * CH + (j16 >> 3)) * 16384 + rrow * 128 +
-                             (((j16 & 7) ^ (rrow & 7)) << 4) + (boff & 15);
-      uint32_t v[kMaxCluster][DPL / 2];
+      for (int m = 0; m < MLQ; ++m) M = fmaxf(M, __uint_as_float(mlr[m].x));
+#pragma unroll
+      for (int off = CPR / 2; off > 0; off >>= 1)
+        M = fmaxf(M, __shfl_xor_sync(kFullMask, M, off, CPR));
+      float w[MLQ];
+      float Lsum = 0.f;
+#pragma unroll
+      for (int m = 0; m < MLQ; ++m) {
+        const float sm = __uint_as_float(mlr[m].y);
+        w[m] = sm > 0.f ? sm * ex2_approx(__uint_as_float(mlr[m].x) - M) : 0.f;
+        Lsum += w[m];
+      }
+#pragma unroll
+      for (int off = CPR / 2; off > 0; off >>= 1) Lsum += __shfl_xor_sync(kFullMask, Lsum, off, CPR);
+      float acc[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) acc[i] = 0.f;
 #pragma unroll
       for (int q = 0; q < kMaxCluster; ++q) {
+        const float wq = __shfl_sync(kFullMask, w[q / CPR], seg0 + q % CPR);
         if (q < cs) {
-          const uint32_t ra = mapa_shared(laddr, q);
-          if (DPL == 4) {
-            const uint2 t = ld_cluster_v2(ra);
-            v[q][0] = t.x;
-            v[q][DPL / 2 - 1] = t.y;
-          } else {
-            v[q][0] = ld_cluster_u32(ra);
+          const uint32_t u[4] = {v[q].x, v[q].y, v[q].z, v[q].w};
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            acc[2 * i] = fmaf(wq, __uint_as_float(u[i] << 16), acc[2 * i]);
+            acc[2 * i + 1] = fmaf(wq, __uint_as_float(u[i] & 0xFFFF0000u), acc[2 * i + 1]);
           }
         }
       }
-      float acc[DPL];
-#pragma unroll
-      for (int i = 0; i < DPL; ++i) acc[i] = 0.f;
-#pragma unroll
-      for (int q = 0; q < kMaxCluster; ++q) {
-        const float wq = __shfl_sync(kFullMask, w, q);
-        if (q < cs) {
-#pragma unroll
-          for (int i = 0; i < DPL / 2; ++i) {
-            acc[2 * i] = fmaf(wq, __uint_as_float(v[q][i] << 16), acc[2 * i]);
-            acc[2 * i + 1] = fmaf(wq, __uint_as_float(v[q][i] & 0xFFFF0000u), acc[2 * i + 1]);
-          }
-        }
+      if (valid) {
+        const bool row_ok = gr < rows && Lsum > 0.f;
+        const float linv = row_ok ? 1.f / Lsum : 0.f;
+        const int64_t orow = (static_cast<int64_t>(b) * a.n_max + gr / pl.group) * a.Hq +
+                             kv * pl.group + gr % pl.group;
+        *reinterpret_cast<uint4*>(a.out + orow * D + q16 * 8) = make_uint4(
+            pack_bf16x2(acc[0] * linv, acc[1] * linv), pack_bf16x2(acc[2] * linv, acc[3] * linv),
+            pack_bf16x2(acc[4] * linv, acc[5] * linv), pack_bf16x2(acc[6] * linv, acc[7] * linv));
+        if (a.lse && q16 == 0) a.lse[orow] = row_ok ? (M + log2f(Lsum)) * kLn2 : 0.f;
       }
-      const bool row_ok = gr < rows && Lsum > 0.f;
-      const float linv = row_ok ? 1.f / Lsum : 0.f;
-      const int64_t orow = (static_cast<int64_t>(b) * a.n_max + gr / pl.group) * a.Hq +
-                           kv * pl.group + gr % pl.group;
-      __nv_bfloat16* dst = a.out + orow * D + lane * DPL;
-      if (DPL == 4) {
-        uint2 o;
-        o.x = pack_bf16x2(acc[0] * linv, acc[1] * linv);
-        o.y = pack_bf16x2(acc[2] * linv, acc[DPL - 1] * linv);
-        *reinterpret_cast<uint2*>(dst) = o;
-      } else {
-        *reinterpret_cast<uint32_t*>(dst) = pack_bf16x2(acc[0] * linv, acc[1] * linv);
-      }
-      if (a.lse && lane == 0) a.lse[orow] = row_ok ? (M + log2f(Lsum)) * kLn2 : 0.f;
     }
   }
   // the peers may still be reading this CTA's shared memory
   __syncwarp();
   cluster_sync();
 }
+
 
 // ---------------------------------------------------------------- host side
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,

@@ -268,13 +268,20 @@ def _attn_inputs(cfg, B, n_nodes, ctx, n_max, device_kv=False, seed=0):
 
 
 def _run_attn(taps, q, kc, vc, bt, ctx, n_nodes, mask, status=None):
-    """kc, vc: logical [num_pages, Hkv, 16, D] caches, packed here."""
+    """kc, vc: logical [num_pages, Hkv, 16, D] caches, packed here. Without a
+    caller-supplied status word, the device status must stay 0 (no page
+    fault, no wait that ran out)."""
     kc = taps.taps_pack_kv_pages(kc)
     vc = taps.taps_pack_kv_pages(vc)
+    own = status is None
+    if own:
+        status = torch.zeros(1, dtype=torch.int32, device=q.device)
     out, lse = taps.taps_tree_verify_attn(q, kc, vc, dt(bt), dt(ctx), dt(n_nodes),
                                           dt(mask.view(np.int32)), int(ctx.max()),
                                           want_lse=True, status=status)
     torch.cuda.synchronize()
+    if own:
+        assert int(status.item()) == 0, int(status.item())
     return out, lse
 
 
@@ -319,6 +326,33 @@ def _sampled_check(q, kc, vc, bt, ctx, nn, mask, out, rng, per_req=6):
         assert np.all(o[b, n:] == 0)
     assert worst <= ATTN_ATOL, worst
     return worst
+
+
+def test_attention_parity_many_tiles(taps):
+    """Every output row against the oracle where each CTA streams several
+    128-token tiles (ctx 4000, 64 nodes: chunks of 4-5 tiles, a ragged last
+    page), so the S/P buffers, the K and V rings and the lazy rescale all
+    wrap around."""
+    cfg = W.CONFIGS["qwen3_8b"]
+    ctx_a = np.array([4000], np.int32)
+    nn = np.array([64], np.int32)
+    q, kc, vc, bt, mask = _attn_inputs(cfg, 1, nn, ctx_a, 64)
+    out, lse = _run_attn(taps, q, kc, vc, bt, ctx_a, nn, mask)
+    ref, ref_lse = O.tree_verify_attn(_f32(q), _f32(kc), _f32(vc), bt, ctx_a, nn, mask)
+    assert np.abs(_f32(out) - ref).max() <= ATTN_ATOL
+    np.testing.assert_allclose(host(lse)[0, :64], ref_lse[0, :64], rtol=1e-4, atol=1e-4)
+
+
+def test_attention_ragged_batch_sampled(taps):
+    """Requests of very different lengths in one launch (one of them a single
+    node on a one-token context), so chunks end inside tiles and some chunks
+    of a cluster are empty."""
+    cfg = W.CONFIGS["qwen3_8b"]
+    ctx = np.array([4000, 1700, 1, 129], np.int32)
+    nn = np.array([64, 17, 1, 40], np.int32)
+    q, kc, vc, bt, mask = _attn_inputs(cfg, 4, nn, ctx, 64, device_kv=True)
+    out, _ = _run_attn(taps, q, kc, vc, bt, ctx, nn, mask)
+    _sampled_check(q, kc, vc, bt, ctx, nn, mask, out, np.random.default_rng(3), per_req=8)
 
 
 @pytest.mark.parametrize("name,n", [("qwen3_8b", 64), ("qwen3_8b", 256), ("qwen3_4b", 64)])
