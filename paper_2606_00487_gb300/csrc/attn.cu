@@ -55,7 +55,7 @@ using namespace sm100;
 constexpr int kRowsPerCta = 128;
 constexpr int kTile = 128;             // tokens per K/V tile
 constexpr int kTilePages = kTile / 16;  // 16-token pages per tile
-constexpr int kKStages = 3;            // K tiles in flight (released after QK)
+constexpr int kKStages = 2;            // K tiles in flight (released after QK)
 constexpr int kVStages = 2;            // V tiles in flight (released after PV)
 constexpr int kSBufs = 3;              // S / P buffers in TMEM
 constexpr int kThreadsTc = 256;
@@ -126,12 +126,18 @@ struct Smem {
   static constexpr uint32_t kQBytes = kChunks * 16384;
   static constexpr uint32_t kK = kQBytes;                     // K ring, TAPS page layout
   static constexpr uint32_t kV = kK + kKStages * kTileBytes;  // V ring
-  static constexpr uint32_t kBar = kV + kVStages * kTileBytes;
-  static constexpr int kNumBars = 2 * kKStages + 2 * kVStages + 2 * kSBufs + 4;
+  // the peers' partial rows of this CTA's slice (cluster launches):
+  // [peer][64-dim half][slice row][128 B], then [peer][slice row] (max, sum);
+  // peers x slice rows <= 150 for every cluster size
+  static constexpr uint32_t kRecv = kV + kVStages * kTileBytes;
+  static constexpr uint32_t kRecvBytes = (152 * (2 * D + 8) + 1023) / 1024 * 1024;
+  static constexpr uint32_t kBar = kRecv + kRecvBytes;
+  static constexpr int kNumBars = 2 * kKStages + 2 * kVStages + 2 * kSBufs + 5;
   static constexpr uint32_t kTmemSlot = kBar + 8 * kNumBars;
   static constexpr uint32_t kAbort = kTmemSlot + 4;
-  static constexpr uint32_t kMl = (kAbort + 4 + 7) / 8 * 8;   // [128] (max, sum) of the rows
-  static constexpr uint32_t kPages = kMl + 8 * kRowsPerCta;   // page ids of this CTA's chunk
+  static constexpr uint32_t kMl = (kAbort + 4 + 15) / 16 * 16;   // [128] (max, sum) of the rows
+  static constexpr uint32_t kStat = kMl + 8 * kRowsPerCta;     // [slice row] (max, sum), cluster-wide
+  static constexpr uint32_t kPages = kStat + 8 * kRowsPerCta;  // page ids of this CTA's chunk
   static constexpr int kMaxChunkPages = kMaxChunkTokens / 16;
   static constexpr uint32_t kBytes = kPages + 4 * kMaxChunkPages;
   // at least half of the SM's shared memory, so that two CTAs (which would
@@ -178,6 +184,7 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
   uint64_t* o_full = pv_done + 1;          // last PV done
   uint64_t* q_full = o_full + 1;
   uint64_t* drain = q_full + 1;
+  uint64_t* recv = drain + 1;              // the peers' partial rows of this CTA's slice landed
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + S::kTmemSlot);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + S::kAbort);
   const int warp = threadIdx.x >> 5;
@@ -247,9 +254,18 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
     mbar_init(o_full, 1);
     mbar_init(q_full, 1);
     mbar_init(drain, 1);
+    mbar_init(recv, 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
+  // cluster exchange geometry: CTA `rank` combines rows [rb, re) of the block
+  const int cs = pl.cs;
+  const uint32_t rank = single ? 0u : cluster_ctarank();
+  const int per = ((kRowsPerCta + cs - 1) / cs + 1) & ~1;   // even: 16-byte (max, sum) pieces
+  const int rb = min(kRowsPerCta, static_cast<int>(rank) * per);
+  const int re = min(kRowsPerCta, rb + per);
+  if (!single && threadIdx.x == 0)
+    mbar_arrive_expect_tx(recv, static_cast<uint32_t>(cs * (re - rb) * (2 * D + 8)));
   // page ids of the whole chunk -> shared memory (producer warp, coalesced);
   // -1 marks a logical page missing from the block table
   int32_t* spages = reinterpret_cast<int32_t*>(smem + S::kPages);
@@ -262,23 +278,10 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  // peers may push into this CTA only once its barriers exist: waited on
+  // before the first push
+  if (!single) cluster_arrive_relaxed();
   const uint32_t tmem = *tmem_slot;
-  // validity of the 64 columns [64 h, 64 h + 64) of tile j: inside the chunk
-  // and on a valid page, 16 bits per page
-  auto tile_cols = [&](int j, int h) -> uint64_t {
-    const int t0 = pos0 + j * kTile + 64 * h;
-    uint64_t cm = 0;
-#pragma unroll
-    for (int p = 0; p < 4; ++p) {
-      const int tp = t0 + 16 * p;
-      if (tp >= pos1) continue;
-      const int pg = spages[j * kTilePages + 4 * h + p];
-      if (pg < 0 || pg >= a.num_pages) continue;
-      const int nv = min(16, pos1 - tp);
-      cm |= (nv == 16 ? 0xFFFFull : ((1ull << nv) - 1)) << (16 * p);
-    }
-    return cm;
-  };
   constexpr uint32_t kOCol = 0;
   auto s_col = [](int u) { return static_cast<uint32_t>(128 + u * 128); };
 
@@ -447,17 +450,31 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
     const uint32_t* mrow = a.mask + (static_cast<int64_t>(b) * a.n_max + node) * a.W;
     float m_used = -INFINITY, l = 0.f;
     bool ok = true;
+    // lane p holds the page id of page p of the next tile, fetched one tile
+    // ahead: shared-memory loads queue behind the tensor core's operand reads
+    auto page_id = [&](int j) {
+      return lane < kTilePages && pos0 + j * kTile + 16 * lane < pos1
+                 ? spages[j * kTilePages + lane] : -1;
+    };
+    int pgn = page_id(0);
     for (int j = 0; j < n_tiles; ++j) {
       if (__any_sync(kFullMask, *abort_flag != 0)) { ok = false; break; }
-      // visible columns of this row in tile j, before waiting for S: these
-      // loads would queue behind the tensor core's shared-memory reads
+      // visible columns of this row in tile j: on a valid page, inside the
+      // chunk, and for tree nodes on the row's ancestor path
+      const uint32_t live = __ballot_sync(kFullMask, pgn >= 0 && pgn < a.num_pages);
+      if (j + 1 < n_tiles) pgn = page_id(j + 1);
       uint64_t vis[2] = {0ull, 0ull};
       if (valid_row) {
         const int t0 = pos0 + j * kTile;
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
-          vis[h] = tile_cols(j, h);
           const int th = t0 + 64 * h;
+#pragma unroll
+          for (int p = 0; p < 4; ++p) {
+            const int nv = min(16, pos1 - (th + 16 * p));
+            if (((live >> (4 * h + p)) & 1u) && nv > 0)
+              vis[h] |= (nv == 16 ? 0xFFFFull : ((1ull << nv) - 1)) << (16 * p);
+          }
           if (th + 64 > C) {
             // columns from i0 on are tree nodes jn = th + i - C
             const int i0 = max(0, C - th);
@@ -584,13 +601,14 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
     }
     reinterpret_cast<float2*>(smem + S::kMl)[r] =
         good ? make_float2(m_used, l) : make_float2(-INFINITY, 0.f);
+    // the staged rows and (max, sum) leave through bulk copies (async proxy)
+    fence_proxy_async_smem();
     if (single) {
       if (a.lse && grow < pl.rows_max) {
         const int64_t orow = (static_cast<int64_t>(b) * a.n_max + grow / pl.group) * a.Hq +
                              kv * pl.group + grow % pl.group;
         a.lse[orow] = good ? (m_used + log2f(l)) * kLn2 : 0.f;
       }
-      fence_proxy_async_smem();
       named_bar_sync(1, 128);
       if (threadIdx.x == 128) {
         for (int c = 0; c < CH; ++c)
@@ -604,102 +622,90 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
 
   __syncwarp();
   tc_fence_before();
-  if (single) {
-    __syncthreads();
-    if (warp == 1) {
-      tc_fence_after();
-      tmem_dealloc(tmem, kTmemCols);
-    }
-    return;
-  }
-  // ---- cluster reduction: CTA `rank` owns a slice of the block's rows and
-  // combines them over every CTA (chunk) of the cluster, reading the peers'
-  // staged rows and (max, sum) through distributed shared memory.
-  cluster_sync();
+  __syncthreads();   // every role is done with TMEM; rows and (max, sum) are staged
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
   }
-  {
-    // a row is read by CPR lanes, 16 bytes each, so one warp instruction
-    // covers RPI rows; (max, sum) reductions stay inside each row's lanes
-    constexpr int CPR = D / 8;
-    constexpr int RPI = 32 / CPR;
-    constexpr int MLQ = (kMaxCluster + CPR - 1) / CPR;
-    constexpr int kWarps = kThreadsTc / 32;
-    const int cs = pl.cs;
-    const uint32_t rank = cluster_ctarank();
-    const int per = (kRowsPerCta + cs - 1) / cs;
-    const int rb = static_cast<int>(rank) * per;
-    const int re = min(kRowsPerCta, rb + per);
-    const int sr = lane / CPR, q16 = lane % CPR;
-    const int seg0 = sr * CPR;
-    for (int base = rb + warp * RPI; base < re; base += kWarps * RPI) {
-      const int rr = base + sr;
-      const int gr = row0 + rr;
-      const bool valid = rr < re && gr < pl.rows_max;
-      // every remote load of the batch is issued before any is used
-      uint2 mlr[MLQ];
-      uint4 v[kMaxCluster];
-#pragma unroll
-      for (int m = 0; m < MLQ; ++m) {
-        const int q = q16 + m * CPR;
-        mlr[m] = (valid && q < cs) ? ld_cluster_v2(mapa_shared(sb + S::kMl + rr * 8, q))
-                                   : make_uint2(__float_as_uint(-INFINITY), 0u);
-      }
-      const uint32_t laddr =
-          sb + S::kQ + (q16 >> 3) * 16384 + rr * 128 + (((q16 & 7) ^ (rr & 7)) << 4);
-#pragma unroll
-      for (int q = 0; q < kMaxCluster; ++q)
-        v[q] = (valid && q < cs) ? ld_cluster_v4(mapa_shared(laddr, q)) : make_uint4(0, 0, 0, 0);
-      float M = -INFINITY;
-#pragma unroll
-      for (int m = 0; m < MLQ; ++m) M = fmaxf(M, __uint_as_float(mlr[m].x));
-#pragma unroll
-      for (int off = CPR / 2; off > 0; off >>= 1)
-        M = fmaxf(M, __shfl_xor_sync(kFullMask, M, off, CPR));
-      float w[MLQ];
-      float Lsum = 0.f;
-#pragma unroll
-      for (int m = 0; m < MLQ; ++m) {
-        const float sm = __uint_as_float(mlr[m].y);
-        w[m] = sm > 0.f ? sm * ex2_approx(__uint_as_float(mlr[m].x) - M) : 0.f;
-        Lsum += w[m];
-      }
-#pragma unroll
-      for (int off = CPR / 2; off > 0; off >>= 1) Lsum += __shfl_xor_sync(kFullMask, Lsum, off, CPR);
-      float acc[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) acc[i] = 0.f;
-#pragma unroll
-      for (int q = 0; q < kMaxCluster; ++q) {
-        const float wq = __shfl_sync(kFullMask, w[q / CPR], seg0 + q % CPR);
-        if (q < cs) {
-          const uint32_t u[4] = {v[q].x, v[q].y, v[q].z, v[q].w};
-#pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            acc[2 * i] = fmaf(wq, __uint_as_float(u[i] << 16), acc[2 * i]);
-            acc[2 * i + 1] = fmaf(wq, __uint_as_float(u[i] & 0xFFFF0000u), acc[2 * i + 1]);
-          }
-        }
-      }
-      if (valid) {
-        const bool row_ok = gr < rows && Lsum > 0.f;
-        const float linv = row_ok ? 1.f / Lsum : 0.f;
-        const int64_t orow = (static_cast<int64_t>(b) * a.n_max + gr / pl.group) * a.Hq +
-                             kv * pl.group + gr % pl.group;
-        *reinterpret_cast<uint4*>(a.out + orow * D + q16 * 8) = make_uint4(
-            pack_bf16x2(acc[0] * linv, acc[1] * linv), pack_bf16x2(acc[2] * linv, acc[3] * linv),
-            pack_bf16x2(acc[4] * linv, acc[5] * linv), pack_bf16x2(acc[6] * linv, acc[7] * linv));
-        if (a.lse && q16 == 0) a.lse[orow] = row_ok ? (M + log2f(Lsum)) * kLn2 : 0.f;
-      }
+  if (single) return;
+  // ---- cluster reduction. Each CTA pushes every peer that peer's slice of
+  // its staged rows and (max, sum) with bulk copies into the peer's receive
+  // buffer as soon as its own rows are staged, then combines its own slice
+  // over the cluster's chunks from shared memory and writes it out.
+  const uint32_t ml_off = static_cast<uint32_t>(cs * CH * per * 128);
+  cluster_wait();
+  if (warp == 0 && lane < cs) {
+    // lane q sends peer q rows [qb, qe) of every 64-dim half and their (max, sum)
+    const int qb = min(kRowsPerCta, lane * per), qe = min(kRowsPerCta, qb + per);
+    if (qe > qb) {
+      const uint32_t dst = mapa_shared(sb + S::kRecv, lane);
+      const uint32_t bar = mapa_shared(smem_u32(recv), lane);
+      for (int c = 0; c < CH; ++c)
+        bulk_copy_to_peer(dst + ((rank * CH + c) * per) * 128, sb + S::kQ + c * 16384 + qb * 128,
+                          (qe - qb) * 128, bar);
+      bulk_copy_to_peer(dst + ml_off + rank * per * 8, sb + S::kMl + qb * 8, (qe - qb) * 8, bar);
     }
   }
-  // the peers may still be reading this CTA's shared memory
+  const bool got = mbar_wait(recv, 0);
+  if (!got && threadIdx.x == 0 && a.status) atomicOr(a.status, TAPS_DEVFAULT_TIMEOUT);
+  // this CTA's slice has landed, so the peers may release what they sent it
+  // (the landing itself was observed on the mbarrier: nothing to release)
   __syncwarp();
-  cluster_sync();
+  cluster_arrive_relaxed();
+  uint8_t* rv = smem + S::kRecv;
+  float2* rml = reinterpret_cast<float2*>(rv + ml_off);
+  float2* stat = reinterpret_cast<float2*>(smem + S::kStat);
+  if (got && threadIdx.x < re - rb) {
+    // per row: the cluster-wide max M, each chunk's weight l_q 2^(m_q - M)
+    // (in place of m_q) and the total L
+    const int i = threadIdx.x;
+    float M = -INFINITY;
+    for (int q = 0; q < cs; ++q) M = fmaxf(M, rml[q * per + i].x);
+    float L = 0.f;
+    for (int q = 0; q < cs; ++q) {
+      const float2 ml = rml[q * per + i];
+      const float w = ml.y > 0.f ? ml.y * ex2_approx(ml.x - M) : 0.f;
+      rml[q * per + i].x = w;
+      L += w;
+    }
+    stat[i] = make_float2(M, L);
+  }
+  __syncthreads();
+  if (got) {
+    for (int e = threadIdx.x; e < (re - rb) * (D / 8); e += kThreadsTc) {
+      const int i = e / (D / 8), q16 = e % (D / 8);
+      const int rr = rb + i, gr = row0 + rr;
+      if (gr >= pl.rows_max) continue;
+      const uint8_t* vp = rv + ((q16 >> 3) * per + i) * 128 + (((q16 & 7) ^ (rr & 7)) << 4);
+      float acc[8];
+#pragma unroll
+      for (int k = 0; k < 8; ++k) acc[k] = 0.f;
+#pragma unroll 4
+      for (int q = 0; q < cs; ++q) {
+        const float w = rml[q * per + i].x;
+        const uint4 v = *reinterpret_cast<const uint4*>(vp + q * CH * per * 128);
+        const uint32_t u[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          acc[2 * k] = fmaf(w, __uint_as_float(u[k] << 16), acc[2 * k]);
+          acc[2 * k + 1] = fmaf(w, __uint_as_float(u[k] & 0xFFFF0000u), acc[2 * k + 1]);
+        }
+      }
+      const float2 st = stat[i];
+      const bool row_ok = gr < rows && st.y > 0.f;
+      const float linv = row_ok ? 1.f / st.y : 0.f;
+      const int64_t orow = (static_cast<int64_t>(b) * a.n_max + gr / pl.group) * a.Hq +
+                           kv * pl.group + gr % pl.group;
+      *reinterpret_cast<uint4*>(a.out + orow * D + q16 * 8) = make_uint4(
+          pack_bf16x2(acc[0] * linv, acc[1] * linv), pack_bf16x2(acc[2] * linv, acc[3] * linv),
+          pack_bf16x2(acc[4] * linv, acc[5] * linv), pack_bf16x2(acc[6] * linv, acc[7] * linv));
+      if (a.lse && q16 == 0) a.lse[orow] = row_ok ? (st.x + log2f(st.y)) * kLn2 : 0.f;
+    }
+  }
+  // every peer has received what this CTA sent it before this CTA exits
+  __syncwarp();
+  cluster_wait();
 }
-
 
 // ---------------------------------------------------------------- host side
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,

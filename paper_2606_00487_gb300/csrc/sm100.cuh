@@ -306,6 +306,26 @@ __device__ __forceinline__ void cluster_sync() {
       "barrier.cluster.arrive.release.aligned;\n\t"
       "barrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
+// Split form of the cluster barrier: every thread of the cluster arrives,
+// then later waits, in this order. The relaxed arrive orders no memory
+// operation of the arriving thread.
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait() {
+  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// Bulk copy of `bytes` (multiple of 16, 16-byte aligned addresses) from this
+// CTA's shared memory to shared memory of a CTA of the cluster; completion is
+// signalled on the mbarrier `bar_cluster` of the destination CTA. Both
+// destination addresses are shared::cluster addresses (see mapa_shared).
+__device__ __forceinline__ void bulk_copy_to_peer(uint32_t dst_cluster, uint32_t src_smem,
+                                                  uint32_t bytes, uint32_t bar_cluster) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+      ::"r"(dst_cluster), "r"(src_smem), "r"(bytes), "r"(bar_cluster)
+      : "memory");
+}
 // Address of the same shared-memory offset in CTA `rank` of the cluster.
 __device__ __forceinline__ uint32_t mapa_shared(uint32_t addr, uint32_t rank) {
   uint32_t r;
