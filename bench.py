@@ -37,6 +37,16 @@ FALLBACK_HBM_GBS = 6800.0
 FALLBACK_BF16_TFLOPS = 1900.0
 
 
+def attn_source_sha256():
+    """Hash of the attention kernel's sources (the kernel and its PTX helpers)."""
+    import hashlib
+    h = hashlib.sha256()
+    for f in ("attn.cu", "sm100.cuh"):
+        with open(os.path.join(ROOT, "paper_2606_00487_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()
+
+
 def load_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -375,7 +385,9 @@ def run_ours(args):
     if os.path.exists(tp):
         try:
             t = json.load(open(tp))
-            if t.get("workload") == cfg.name and t.get("n_max") == cfg.n_max:
+            # counters taken on another version of the kernel do not count
+            if (t.get("workload") == cfg.name and t.get("n_max") == cfg.n_max
+                    and t.get("source_sha256") == attn_source_sha256()):
                 traffic = t.get("bytes_per_launch")
         except Exception:
             traffic = None
