@@ -191,27 +191,76 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
   const int lane = threadIdx.x & 31;
 
   // ---- set-up that reads no input: may overlap the previous grid's tail
-  if (threadIdx.x == 0) prefetch_tensormap(&maps.q);
-  if (warp == 1) {
-    tmem_alloc(tmem_slot, kTmemCols);
-    tmem_relinquish();
-  }
-  pdl_wait();
-
   const Plan& pl = a.plan;
   const int b = blockIdx.z;
   const int kv = blockIdx.y / pl.m_blocks;
   const int mb = blockIdx.y % pl.m_blocks;
   const int split = blockIdx.x;
+  const int row0 = mb * kRowsPerCta;
+  const int pos0 = split * pl.chunk_len;
+  const bool single = pl.cs == 1;
+  // cluster exchange geometry: CTA `rank` combines rows [rb, re) of the block
+  const int cs = pl.cs;
+  const uint32_t rank = single ? 0u : cluster_ctarank();
+  const int per = ((kRowsPerCta + cs - 1) / cs + 1) & ~1;   // even: 16-byte (max, sum) pieces
+  const int rb = min(kRowsPerCta, static_cast<int>(rank) * per);
+  const int re = min(kRowsPerCta, rb + per);
+  if (threadIdx.x == 0) {
+    prefetch_tensormap(&maps.q);
+    for (int s = 0; s < kKStages; ++s) {
+      mbar_init(&k_full[s], 1);
+      mbar_init(&k_empty[s], 1);
+    }
+    for (int s = 0; s < kVStages; ++s) {
+      mbar_init(&v_full[s], 1);
+      mbar_init(&v_empty[s], 1);
+    }
+    for (int u = 0; u < kSBufs; ++u) {
+      mbar_init(&s_full[u], 1);
+      mbar_init(&p_full[u], 4);
+    }
+    mbar_init(pv_done, 1);
+    mbar_init(o_full, 1);
+    mbar_init(q_full, 1);
+    mbar_init(drain, 1);
+    mbar_init(recv, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+    if (!single) mbar_arrive_expect_tx(recv, static_cast<uint32_t>(cs * (re - rb) * (2 * D + 8)));
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, kTmemCols);
+    tmem_relinquish();
+  }
+  __syncthreads();   // barriers initialised
+  pdl_wait();
+
+  // ---- inputs. The request's lengths and the chunk's page ids are
+  // requested together; then Q and each producer's first tile leave at once,
+  // before the CTA-wide barrier.
+  // page ids of the chunk -> shared memory (warp 0, coalesced; -1 marks a
+  // logical page missing from the block table); lane p of warps 0 and 2 keeps
+  // the id of page p of the first tile
+  int32_t* spages = reinterpret_cast<int32_t*>(smem + S::kPages);
+  const int32_t* bt = a.block_table + static_cast<int64_t>(b) * a.max_pages;
+  const int lp0 = pos0 >> 4;
+  int pg0 = -1;
+  if (warp == 0) {
+    const int npg = (pl.chunk_len + 15) >> 4;   // a full chunk's pages; the unused tail is harmless
+    for (int i = lane; i < npg; i += 32) {
+      const int id = lp0 + i < a.max_pages ? bt[lp0 + i] : -1;
+      spages[i] = id;
+      if (i == lane) pg0 = id;
+    }
+  } else if (warp == 2 && lane < kTilePages) {
+    pg0 = lp0 + lane < a.max_pages ? bt[lp0 + lane] : -1;
+  }
   const int n = min(max(a.n_nodes[b], 0), a.n_max);
   const int C = a.ctx_len[b];
   const int total = C + n;
   const int rows = n * pl.group;
-  const int row0 = mb * kRowsPerCta;
-  const int pos0 = split * pl.chunk_len;
   const int pos1 = min(pos0 + pl.chunk_len, total);
   const int n_tiles = pos1 > pos0 ? (pos1 - pos0 + kTile - 1) / kTile : 0;
-  const bool single = pl.cs == 1;
 
   if (row0 >= rows) {
     // no row of this block is live (the same for every CTA of a cluster): the
@@ -237,44 +286,33 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
     return;
   }
 
-  if (threadIdx.x == 0) {
-    for (int s = 0; s < kKStages; ++s) {
-      mbar_init(&k_full[s], 1);
-      mbar_init(&k_empty[s], 1);
+  // the first K or V tile: lane p copies page p
+  const uint64_t policy = l2_evict_first_policy();
+  auto issue_tile = [&](bool is_k, int j, int pg) {
+    uint64_t* full = is_k ? k_full : v_full;
+    const int s = j % (is_k ? kKStages : kVStages);
+    const bool in = lane < kTilePages && pos0 + j * kTile + 16 * lane < pos1;
+    const bool valid = in && pg >= 0 && pg < a.num_pages;
+    if (is_k && in && !valid && a.status) atomicOr(a.status, TAPS_DEVFAULT_PAGE);
+    const uint32_t vm = __ballot_sync(kFullMask, valid);
+    if (lane == 0) mbar_arrive_expect_tx(&full[s], __popc(vm) * S::kPageBytes);
+    __syncwarp();
+    if (valid) {
+      const int64_t blk = (static_cast<int64_t>(pg) * a.Hkv + kv) * (16 * D);
+      bulk_load(sb + (is_k ? S::kK : S::kV) + s * S::kTileBytes + lane * S::kPageBytes,
+                (is_k ? a.k : a.v) + blk, S::kPageBytes, &full[s], policy);
     }
-    for (int s = 0; s < kVStages; ++s) {
-      mbar_init(&v_full[s], 1);
-      mbar_init(&v_empty[s], 1);
-    }
-    for (int u = 0; u < kSBufs; ++u) {
-      mbar_init(&s_full[u], 1);
-      mbar_init(&p_full[u], 4);
-    }
-    mbar_init(pv_done, 1);
-    mbar_init(o_full, 1);
-    mbar_init(q_full, 1);
-    mbar_init(drain, 1);
-    mbar_init(recv, 1);
-    *abort_flag = 0;
-    fence_mbar_init();
+  };
+  if (n_tiles > 0 && threadIdx.x == 0) {
+    // Q rows of this block: one box of (64 dims, group heads, 128/group
+    // nodes) per 64-dim half; nodes past n_max read as zeros. (Not for an
+    // empty chunk, whose epilogue stages its zero rows in the Q buffer.)
+    mbar_arrive_expect_tx(q_full, static_cast<uint32_t>(CH * 16384));
+    for (int c = 0; c < CH; ++c)
+      tma_load_4d(sb + S::kQ + c * 16384, &maps.q, q_full, c * 64, kv * pl.group,
+                  row0 / pl.group, b);
   }
-  // cluster exchange geometry: CTA `rank` combines rows [rb, re) of the block
-  const int cs = pl.cs;
-  const uint32_t rank = single ? 0u : cluster_ctarank();
-  const int per = ((kRowsPerCta + cs - 1) / cs + 1) & ~1;   // even: 16-byte (max, sum) pieces
-  const int rb = min(kRowsPerCta, static_cast<int>(rank) * per);
-  const int re = min(kRowsPerCta, rb + per);
-  if (!single && threadIdx.x == 0)
-    mbar_arrive_expect_tx(recv, static_cast<uint32_t>(cs * (re - rb) * (2 * D + 8)));
-  // page ids of the whole chunk -> shared memory (producer warp, coalesced);
-  // -1 marks a logical page missing from the block table
-  int32_t* spages = reinterpret_cast<int32_t*>(smem + S::kPages);
-  if (warp == 0) {
-    const int32_t* bt = a.block_table + static_cast<int64_t>(b) * a.max_pages;
-    const int lp0 = pos0 >> 4;
-    const int npg = (pos1 - pos0 + 15) >> 4;
-    for (int i = lane; i < npg; i += 32) spages[i] = lp0 + i < a.max_pages ? bt[lp0 + i] : -1;
-  }
+  if (n_tiles > 0 && (warp == 0 || warp == 2)) issue_tile(warp == 0, 0, pg0);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -290,45 +328,24 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
     // below contributes zero rows with an empty softmax
   } else if (warp == 0 || warp == 2) {
     // ------------------------------------------------------------ TMA producers
-    // warp 0 streams Q and the K tiles, warp 2 the V tiles, each into its own
-    // ring, so neither producer's wait stalls the other. Lane p handles page
-    // p of a tile: its page id is fetched one tile ahead, and the eight bulk
-    // copies of a tile leave in one warp instruction.
+    // warp 0 streams the K tiles, warp 2 the V tiles, each into its own ring,
+    // so neither producer's wait stalls the other. Lane p handles page p of a
+    // tile, with its page id fetched one tile ahead; tile 0 left above.
     const bool is_k = warp == 0;
     const int nst = is_k ? kKStages : kVStages;
     uint64_t* full = is_k ? k_full : v_full;
     uint64_t* empty = is_k ? k_empty : v_empty;
-    const __nv_bfloat16* cache = is_k ? a.k : a.v;
-    const uint32_t ring = sb + (is_k ? S::kK : S::kV);
-    const uint64_t policy = l2_evict_first_policy();
-    if (is_k && lane == 0) {
-      // Q rows of this block first: one box of (64 dims, group heads,
-      // 128/group nodes) per 64-dim half; nodes past n_max read as zeros
-      mbar_arrive_expect_tx(q_full, static_cast<uint32_t>(CH * 16384));
-      for (int c = 0; c < CH; ++c)
-        tma_load_4d(sb + S::kQ + c * 16384, &maps.q, q_full, c * 64, kv * pl.group,
-                    row0 / pl.group, b);
-    }
     auto in_chunk = [&](int j) { return lane < kTilePages && pos0 + j * kTile + 16 * lane < pos1; };
-    int pg = in_chunk(0) ? spages[lane] : -1;
-    int issued = 0;
-    for (int j = 0; j < n_tiles; ++j) {
+    int pg = n_tiles > 1 && in_chunk(1) ? spages[kTilePages + lane] : -1;
+    int issued = 1;
+    for (int j = 1; j < n_tiles; ++j) {
       if (__any_sync(kFullMask, *abort_flag != 0)) break;
       const int s = j % nst;
       if (j >= nst && !__all_sync(kFullMask, mbar_wait(&empty[s], ((j / nst) - 1) & 1))) {
         if (lane == 0) set_fault(abort_flag, a.status, TAPS_DEVFAULT_TIMEOUT);
         break;
       }
-      const bool valid = pg >= 0 && pg < a.num_pages;
-      if (is_k && in_chunk(j) && !valid && a.status) atomicOr(a.status, TAPS_DEVFAULT_PAGE);
-      const uint32_t vm = __ballot_sync(kFullMask, valid);
-      if (lane == 0) mbar_arrive_expect_tx(&full[s], __popc(vm) * S::kPageBytes);
-      __syncwarp();
-      if (valid) {
-        const int64_t blk = (static_cast<int64_t>(pg) * a.Hkv + kv) * (16 * D);
-        bulk_load(ring + s * S::kTileBytes + lane * S::kPageBytes, cache + blk, S::kPageBytes,
-                  &full[s], policy);
-      }
+      issue_tile(is_k, j, pg);
       issued = j + 1;
       if (j + 1 < n_tiles) pg = in_chunk(j + 1) ? spages[(j + 1) * kTilePages + lane] : -1;
     }
