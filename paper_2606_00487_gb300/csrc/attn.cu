@@ -238,21 +238,17 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
   // ---- inputs. The request's lengths and the chunk's page ids are
   // requested together; then Q and each producer's first tile leave at once,
   // before the CTA-wide barrier.
-  // page ids of the chunk -> shared memory (warp 0, coalesced; -1 marks a
-  // logical page missing from the block table); lane p of warps 0 and 2 keeps
-  // the id of page p of the first tile
+  // page ids of the chunk -> shared memory (warp 3, coalesced; -1 marks a
+  // logical page missing from the block table); lane p of the producer warps
+  // 0 and 2 reads the id of page p of the first tile for itself
   int32_t* spages = reinterpret_cast<int32_t*>(smem + S::kPages);
   const int32_t* bt = a.block_table + static_cast<int64_t>(b) * a.max_pages;
   const int lp0 = pos0 >> 4;
   int pg0 = -1;
-  if (warp == 0) {
+  if (warp == 3) {
     const int npg = (pl.chunk_len + 15) >> 4;   // a full chunk's pages; the unused tail is harmless
-    for (int i = lane; i < npg; i += 32) {
-      const int id = lp0 + i < a.max_pages ? bt[lp0 + i] : -1;
-      spages[i] = id;
-      if (i == lane) pg0 = id;
-    }
-  } else if (warp == 2 && lane < kTilePages) {
+    for (int i = lane; i < npg; i += 32) spages[i] = lp0 + i < a.max_pages ? bt[lp0 + i] : -1;
+  } else if ((warp == 0 || warp == 2) && lane < kTilePages) {
     pg0 = lp0 + lane < a.max_pages ? bt[lp0 + lane] : -1;
   }
   const int n = min(max(a.n_nodes[b], 0), a.n_max);
@@ -303,10 +299,10 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
                 (is_k ? a.k : a.v) + blk, S::kPageBytes, &full[s], policy);
     }
   };
-  if (n_tiles > 0 && threadIdx.x == 0) {
-    // Q rows of this block: one box of (64 dims, group heads, 128/group
-    // nodes) per 64-dim half; nodes past n_max read as zeros. (Not for an
-    // empty chunk, whose epilogue stages its zero rows in the Q buffer.)
+  if (n_tiles > 0 && threadIdx.x == 96) {
+    // (warp 3) Q rows of this block: one box of (64 dims, group heads,
+    // 128/group nodes) per 64-dim half; nodes past n_max read as zeros. (Not
+    // for an empty chunk, whose epilogue stages its zero rows in the Q buffer.)
     mbar_arrive_expect_tx(q_full, static_cast<uint32_t>(CH * 16384));
     for (int c = 0; c < CH; ++c)
       tma_load_4d(sb + S::kQ + c * 16384, &maps.q, q_full, c * 64, kv * pl.group,
@@ -515,11 +511,13 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
         for (int i = 0; i < 128; ++i)
           if (!((vis[i >> 6] >> (i & 63)) & 1ull)) sv[i] = 0xFF800000u;   // -inf
       }
+      // row max: eight chains of three-input maxima
       float mx[8];
 #pragma unroll
       for (int k = 0; k < 8; ++k) mx[k] = __uint_as_float(sv[k]);
 #pragma unroll
-      for (int i = 8; i < 128; ++i) mx[i & 7] = fmaxf(mx[i & 7], __uint_as_float(sv[i]));
+      for (int i = 8; i < 128; i += 2)
+        mx[(i >> 1) & 7] = max3f(mx[(i >> 1) & 7], __uint_as_float(sv[i]), __uint_as_float(sv[i + 1]));
       const float tmax =
           fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
                 fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7]))) * scale;
@@ -531,27 +529,34 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
         alpha = (m_used == -INFINITY) ? 0.f : ex2_approx(m_used - m_new);
         m_used = m_new;
       }
-      float acc[8];
-#pragma unroll
-      for (int k = 0; k < 8; ++k) acc[k] = 0.f;
       // P over the first 64 columns of this S buffer (the row's S is in
-      // registers), in two halves of 32 columns
+      // registers), in two halves of 32 columns: x = s * scale - m for two
+      // columns per packed FMA, 2^x on the SFU, bf16 pairs, packed row sums
       const float nm = m_used == -INFINITY ? 0.f : -m_used;
       const bool any = m_used != -INFINITY;
+      const uint64_t scale2 = f32x2(scale, scale), nm2 = f32x2(nm, nm);
+      uint64_t acc2[4] = {0ull, 0ull, 0ull, 0ull};
 #pragma unroll
       for (int h = 0; h < 2; ++h) {
         uint32_t pk[32];
 #pragma unroll
         for (int i = 0; i < 32; ++i) {
-          const float p0 = any ? ex2_approx(fmaf(__uint_as_float(sv[64 * h + 2 * i]), scale, nm)) : 0.f;
-          const float p1 = any ? ex2_approx(fmaf(__uint_as_float(sv[64 * h + 2 * i + 1]), scale, nm)) : 0.f;
+          const uint64_t x = fma_f32x2(
+              f32x2(__uint_as_float(sv[64 * h + 2 * i]), __uint_as_float(sv[64 * h + 2 * i + 1])),
+              scale2, nm2);
+          float x0, x1;
+          f32x2_split(x, x0, x1);
+          const float p0 = any ? ex2_approx(x0) : 0.f;
+          const float p1 = any ? ex2_approx(x1) : 0.f;
           pk[i] = pack_bf16x2(p0, p1);
-          acc[i & 7] += p0 + p1;
+          acc2[i & 3] = add_f32x2(acc2[i & 3], f32x2(p0, p1));
         }
         tmem_st32(lane_base + s_col(u) + 32 * h, pk);
       }
-      const float psum = ((acc[0] + acc[1]) + (acc[2] + acc[3])) +
-                         ((acc[4] + acc[5]) + (acc[6] + acc[7]));
+      float a0, a1, a2, a3;
+      f32x2_split(add_f32x2(acc2[0], acc2[1]), a0, a1);
+      f32x2_split(add_f32x2(acc2[2], acc2[3]), a2, a3);
+      const float psum = (a0 + a1) + (a2 + a3);
       l = l * alpha + psum;
       // a grown max rescales O before P of this tile is released; the PV of
       // the previous tile may still be running, so wait for it first
