@@ -375,14 +375,28 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
       __syncwarp();
     }
     bool o_started = false;   // O holds a first product
-    auto page_id = [&](int j) {
-      return lane < kTilePages && pos0 + j * kTile + 16 * lane < pos1
-                 ? spages[j * kTilePages + lane] : -1;
-    };
-    int pgv = page_id(0);
+    // Pages holding a valid token, one byte per tile of the chunk (at most
+    // kMaxChunkTokens / kTile = 256 tiles): lane l keeps tiles l, l + 32, ...
+    // Read once here, while Q and the first tiles load, so that no
+    // shared-memory load (queued behind the tensor core's operand reads)
+    // sits between two bursts.
+    uint64_t live8 = 0;
+    for (int t = lane; t < n_tiles; t += 32) {
+      uint32_t m = 0;
+      for (int p = 0; p < kTilePages; ++p) {
+        if (pos0 + t * kTile + 16 * p >= pos1) break;
+        const int pg = spages[t * kTilePages + p];
+        if (pg >= 0 && pg < a.num_pages) m |= 1u << p;
+      }
+      live8 |= static_cast<uint64_t>(m) << (8 * (t >> 5));
+    }
+    // the page cut by the end of the sequence, if any: its rows past the end
+    // are zeroed so that P = 0 never meets stale (possibly non-finite) data
+    const int cut_tile = (pos1 & 15) ? (pos1 - 1 - pos0) / kTile : -1;
+    const int cut_page = (pos1 & 15) ? ((pos1 - 1 - pos0) % kTile) / 16 : 0;
     // burst j: PV of tile j (after its softmax) alternating with QK of tile j+2
+    // (no abort-flag poll here: every wait is bounded)
     for (int j = 0; ok && j < n_tiles; ++j) {
-      if (__any_sync(kFullMask, *abort_flag != 0)) break;
       const int jn = j + 2;
       const bool has_qk = jn < n_tiles;
       const int sv = j % kVStages;
@@ -390,18 +404,11 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
         ok = false;
         break;
       }
-      // pages of tile j holding a valid token (lane p: page p, id fetched
-      // during the previous burst), and the page cut by the end of the
-      // sequence, whose rows past the end are zeroed so that P = 0 never
-      // meets stale (possibly non-finite) data
-      const int tp = pos0 + j * kTile + 16 * lane;
-      const bool live = pgv >= 0 && pgv < a.num_pages;
-      const uint32_t page_live = __ballot_sync(kFullMask, live);
-      const uint32_t cut = __ballot_sync(kFullMask, live && pos1 - tp < 16);
-      if (cut) {
-        const int p = __ffs(cut) - 1;
-        const int nv = __shfl_sync(kFullMask, pos1 - tp, p);
-        uint8_t* pb = smem + S::kV + sv * S::kTileBytes + p * S::kPageBytes;
+      const uint32_t page_live =
+          static_cast<uint32_t>(__shfl_sync(kFullMask, live8, j & 31) >> (8 * (j >> 5))) & 0xFFu;
+      if (j == cut_tile && ((page_live >> cut_page) & 1u)) {
+        const int nv = pos1 & 15;
+        uint8_t* pb = smem + S::kV + sv * S::kTileBytes + cut_page * S::kPageBytes;
         for (int e = lane; e < 16 * 8 * CH; e += 32) {
           const int w = e / (8 * CH), c = (e / 8) % CH, q16 = e % 8;
           if (w >= nv)
@@ -442,7 +449,6 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
         if (j == n_tiles - 1) mma_commit(o_full);
       }
       __syncwarp();
-      if (j + 1 < n_tiles) pgv = page_id(j + 1);
     }
     if (!ok && lane == 0) set_fault(abort_flag, a.status, TAPS_DEVFAULT_TIMEOUT);
     // every MMA issued by this warp completes before TMEM is released
