@@ -400,9 +400,24 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
       const int jn = j + 2;
       const bool has_qk = jn < n_tiles;
       const int sv = j % kVStages;
-      if (!__all_sync(kFullMask, mbar_wait(&v_full[sv], (j / kVStages) & 1))) {
-        ok = false;
-        break;
+      // V tile j, K tile j+2 and P of tile j: the three barriers are tested
+      // back to back (their latencies overlap), and only one that has not
+      // completed yet is then waited on
+      {
+        uint64_t* bv = &v_full[sv];
+        uint64_t* bk = &k_full[jn % kKStages];
+        uint64_t* bp = &p_full[j % kSBufs];
+        const uint32_t qv = (j / kVStages) & 1, qk = (jn / kKStages) & 1, qp = (j / kSBufs) & 1;
+        bool wv = mbar_try_wait(bv, qv);
+        bool wk = !has_qk || mbar_try_wait(bk, qk);
+        bool wp = mbar_try_wait(bp, qp);
+        if (!wv) wv = mbar_wait(bv, qv);
+        if (!wk) wk = mbar_wait(bk, qk);
+        if (!wp) wp = mbar_wait(bp, qp);
+        if (!__all_sync(kFullMask, wv && wk && wp)) {
+          ok = false;
+          break;
+        }
       }
       const uint32_t page_live =
           static_cast<uint32_t>(__shfl_sync(kFullMask, live8, j & 31) >> (8 * (j >> 5))) & 0xFFu;
@@ -418,15 +433,6 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
         fence_proxy_async_smem();
       }
       __syncwarp();
-      if (has_qk &&
-          !__all_sync(kFullMask, mbar_wait(&k_full[jn % kKStages], (jn / kKStages) & 1))) {
-        ok = false;
-        break;
-      }
-      if (!__all_sync(kFullMask, mbar_wait(&p_full[j % kSBufs], (j / kSBufs) & 1))) {
-        ok = false;
-        break;
-      }
       if (lane == 0) {
         tc_fence_after();
         const uint32_t vb = sb + S::kV + sv * S::kTileBytes;
