@@ -338,6 +338,35 @@ def run_ours(args):
     torch.cuda.synchronize()
     one_layer_us = f0.elapsed_time(f1) / reps * 1e3
 
+    # ---- per-stage time: each stage alone as a graph, replayed back to back
+    q0, k0, v0, b0 = layers[0]
+    stage_fns = {
+        "s1_topk": lambda: taps.taps_topk_marginals(
+            logits, cfg.K, out=(r.ids, r.logp, r.lse, r.entropy), ws=r.ws_topk),
+        "s2_score": lambda: taps.taps_score_reach(root, r.ids, r.logp, r.entropy, r.scorer,
+                                                  out=r.q_cond),
+        "s3_select": lambda: taps.taps_select_subtree(r.q_cond, r.ids, root, ctx, r.lambda1,
+                                                      r.lambda2, r.tau, r.n_max, out=r.sel),
+        "s4_mask": lambda: taps.taps_build_tree_mask(r.sel["parent"], r.sel["n_nodes"],
+                                                     out=r.mask),
+        "s5_attention_one_layer": lambda: r.verify_layer(q0, k0, v0, b0, ctx, outs[0]),
+        "s6_accept": lambda: r.accept(target),
+    }
+    stage_us = {}
+    for name, fn in stage_fns.items():
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=s):
+            fn()
+        for _ in range(3):
+            g.replay()
+        torch.cuda.synchronize()
+        f0.record(stream)
+        for _ in range(reps):
+            g.replay()
+        f1.record(stream)
+        torch.cuda.synchronize()
+        stage_us[name] = round(f0.elapsed_time(f1) / reps * 1e3, 2)
+
     # ---- end to end through the public API with host buffers
     e2e = None
     if not args.no_e2e:
@@ -416,6 +445,7 @@ def run_ours(args):
                    "select_plus_one_layer_round_us": round(one_layer_us, 2),
                    "attention_stage_us_per_round": round(attn_ms * 1e3, 2)},
         "roofline": roofline,
+        "stage_us": stage_us,
         "e2e": e2e,
         "gpu_launches": launches,
         "clocks": clk,
