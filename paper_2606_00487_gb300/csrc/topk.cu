@@ -5,11 +5,13 @@
 // `chunks` contiguous slices, one CTA each, so that a batch-1 round still
 // spreads over every SM. A CTA reads its slice with 16-byte vector loads,
 // keeps per-thread running statistics (max, sum of exponentials, sum of
-// exponential-weighted offsets for the entropy) and a per-thread sorted top-K
-// list of 64-bit keys (ordered logit << 32 | ~token id), merges them with warp
-// redux operations, and writes one partial record. The last CTA of a row (an
-// atomic ticket, reset after use) merges the partials and writes the row's
-// outputs. No CTA waits on another.
+// exponential-weighted offsets for the entropy) and, per warp, the running
+// top-K of 64-bit keys (ordered logit << 32 | ~token id) in registers: each
+// tile of two vectors per lane is merged in by K rounds of a warp maximum,
+// and skipped when no key beats the current K-th. The CTA's warps merge by
+// rank into one partial record. The last CTA of a row (an atomic ticket,
+// reset after use) merges the partials by rank and writes the row's outputs.
+// No CTA waits on another.
 #include <algorithm>
 #include <mutex>
 
@@ -38,7 +40,9 @@ Plan make_plan(int B, int L, int V, int K) {
   Plan p;
   p.rows = B * L;
   p.kp = round_kp(K);
-  int want = (4 * kTargetSms + p.rows - 1) / p.rows;
+  // two CTAs per SM: the 256-thread CTAs hold about 80 registers per thread,
+  // so three fit an SM, and one wave of two per SM avoids a second wave
+  int want = (2 * kTargetSms + p.rows - 1) / p.rows;
   int maxc = std::max(1, V / 2048);
   p.chunks = std::max(1, std::min(want, std::min(maxc, kMaxChunks)));
   return p;
@@ -67,6 +71,12 @@ WsLayout ws_layout(const Plan& p) {
   return w;
 }
 
+__device__ __forceinline__ float ex2f(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 // Running softmax statistics in log2 units: m2 = max x*log2(e),
 // z = sum 2^(x2 - m2), t2 = sum 2^(x2 - m2) * (x2 - m2).
 struct Stats {
@@ -77,7 +87,7 @@ __device__ __forceinline__ void stats_raise(Stats& s, float m2_new) {
   if (m2_new > s.m2) {
     if (s.z > 0.f) {
       float dm = s.m2 - m2_new;
-      float sc = exp2f(dm);
+      float sc = ex2f(dm);
       s.t2 = sc * fmaf(s.z, dm, s.t2);
       s.z *= sc;
     }
@@ -88,7 +98,7 @@ __device__ __forceinline__ void stats_raise(Stats& s, float m2_new) {
 __device__ __forceinline__ void stats_add(Stats& s, float x2) {
   if (x2 > -INFINITY) {
     float dx = x2 - s.m2;
-    float e = exp2f(dx);
+    float e = ex2f(dx);
     s.z += e;
     s.t2 = fmaf(e, dx, s.t2);
   }
@@ -99,30 +109,17 @@ __device__ __forceinline__ Stats stats_merge(Stats a, Stats b) {
   Stats r{m, 0.f, 0.f};
   if (a.z > 0.f) {
     float d = a.m2 - m;
-    float s = exp2f(d);
+    float s = ex2f(d);
     r.z += s * a.z;
     r.t2 += s * fmaf(a.z, d, a.t2);
   }
   if (b.z > 0.f) {
     float d = b.m2 - m;
-    float s = exp2f(d);
+    float s = ex2f(d);
     r.z += s * b.z;
     r.t2 += s * fmaf(b.z, d, b.t2);
   }
   return r;
-}
-
-template <int KP>
-__device__ __forceinline__ void list_insert(uint64_t (&lst)[KP], uint64_t key) {
-  if (key <= lst[KP - 1]) return;
-#pragma unroll
-  for (int i = 0; i < KP; ++i) {
-    if (key > lst[i]) {
-      uint64_t t = lst[i];
-      lst[i] = key;
-      key = t;
-    }
-  }
 }
 
 __device__ __forceinline__ uint64_t make_key(float x, uint32_t id) {
@@ -138,29 +135,25 @@ __device__ __forceinline__ float to_f32<__nv_bfloat16>(__nv_bfloat16 v) {
   return __bfloat162float(v);
 }
 
-template <int KP, typename T>
-__device__ __forceinline__ void consume(float x, uint32_t id, Stats& st, uint64_t (&lst)[KP]) {
-  stats_add(st, x * kLog2e);
-  list_insert<KP>(lst, make_key(x, id));
-}
-
-// Merge KP rounds over `count` unsorted keys in shared memory (one warp).
+// The KP largest of n <= 256 keys in shared memory (unique, 0 = none), by one
+// warp: each lane holds eight of them in registers, then KP rounds of a warp
+// maximum. Writes out[0, KP) descending (zero-padded).
 template <int KP>
-__device__ void warp_select_smem(uint64_t* cand, int count, uint64_t* out, int lane) {
+__device__ void warp_top(const uint64_t* cand, int n, uint64_t* out, int lane) {
+  uint64_t c[8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) c[i] = lane + 32 * i < n ? cand[lane + 32 * i] : 0ull;
+#pragma unroll 1
   for (int r = 0; r < KP; ++r) {
     uint64_t mine = 0;
-    int mi = -1;
-    for (int i = lane; i < count; i += 32) {
-      uint64_t v = cand[i];
-      if (v > mine) {
-        mine = v;
-        mi = i;
-      }
-    }
-    uint64_t best = warp_max_u64(mine);
-    if (best != 0 && mine == best) cand[mi] = 0;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) mine = c[i] > mine ? c[i] : mine;
+    const uint64_t best = warp_max_u64(mine);
     if (lane == 0) out[r] = best;
-    __syncwarp();
+    if (best != 0 && mine == best) {
+#pragma unroll
+      for (int i = 0; i < 8; ++i) c[i] = c[i] == best ? 0ull : c[i];
+    }
   }
 }
 
@@ -203,6 +196,7 @@ topk_marginals_kernel(const T* __restrict__ logits, int64_t row_stride, int V, i
   constexpr int VE = 16 / sizeof(T);
   __shared__ uint64_t s_cand[kMaxChunks * 32];
   __shared__ uint64_t s_top[32];
+  __shared__ uint64_t s_part[kWarps * 32];
   __shared__ Stats s_wstats[kWarps];
   __shared__ int s_last;
 
@@ -214,29 +208,88 @@ topk_marginals_kernel(const T* __restrict__ logits, int64_t row_stride, int V, i
   const T* x = logits + static_cast<int64_t>(row) * row_stride;
 
   Stats st{-INFINITY, 0.f, 0.f};
-  uint64_t lst[KP];
+  // The warp's running top-KP keys: lane r < KP holds the r-th largest so far;
+  // kth is the KP-th largest (0 while fewer than KP elements were seen).
+  uint64_t run = 0, kth = 0;
+  // Merge one tile (EPT keys per lane, 0 = none) into the running top-KP. A
+  // tile with no key above kth changes nothing and is skipped. Otherwise tk =
+  // the KP-th largest of the 32 lane maxima: at least KP keys of the tile are
+  // >= tk, so its top-KP lies among them. Each lane keeps those (and above kth)
+  // in four registers, and KP rounds of a 64-bit warp maximum run over them
+  // and the running list; a lane with more than four (heavy ties) sends the
+  // tile through the same rounds over all of its keys instead.
+  constexpr int EPT = 2 * VE;
+  auto merge_tile = [&](uint64_t (&k)[EPT]) {
+    uint64_t lm = 0;
 #pragma unroll
-  for (int i = 0; i < KP; ++i) lst[i] = 0;
+    for (int i = 0; i < EPT; ++i) lm = k[i] > lm ? k[i] : lm;
+    if (!__any_sync(kFullMask, lm > kth)) return;
+    int rank = 0;   // lane maxima above this lane's (keys are unique, 0 = none)
+#pragma unroll
+    for (int l = 0; l < 32; ++l) rank += __shfl_sync(kFullMask, lm, l) > lm ? 1 : 0;
+    const uint32_t at = __ballot_sync(kFullMask, lm != 0 && rank == KP - 1);
+    const uint64_t tk = at ? __shfl_sync(kFullMask, lm, __ffs(at) - 1) : 0ull;
+    uint64_t c[4] = {0ull, 0ull, 0ull, 0ull};
+    int cnt = 0;
+#pragma unroll
+    for (int i = 0; i < EPT; ++i) {
+      if (k[i] >= tk && k[i] > kth) {
+        c[3] = c[2];
+        c[2] = c[1];
+        c[1] = c[0];
+        c[0] = k[i];
+        ++cnt;
+      }
+    }
+    const bool wide = __any_sync(kFullMask, cnt > 4);
+    uint64_t nrun = 0;
+#pragma unroll 1
+    for (int r = 0; r < KP; ++r) {
+      uint64_t mine = run;
+      if (wide) {
+#pragma unroll
+        for (int i = 0; i < EPT; ++i) mine = k[i] > mine ? k[i] : mine;
+      } else {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) mine = c[i] > mine ? c[i] : mine;
+      }
+      const uint64_t best = warp_max_u64(mine);
+      if (lane == r) nrun = best;
+      if (best != 0 && mine == best) {
+        if (run == best) run = 0;
+        if (wide) {
+#pragma unroll
+          for (int i = 0; i < EPT; ++i) k[i] = k[i] == best ? 0ull : k[i];
+        } else {
+#pragma unroll
+          for (int i = 0; i < 4; ++i) c[i] = c[i] == best ? 0ull : c[i];
+        }
+      }
+    }
+    run = nrun;
+    kth = __shfl_sync(kFullMask, nrun, KP - 1);
+  };
 
   if (vec_ok) {
+    // two 16-byte vectors per thread and tile
     const int nvec = V / VE;
     const int per = (nvec + chunks - 1) / chunks;
     const int v0 = chunk * per;
     const int v1 = min(nvec, v0 + per);
     const uint4* xv = reinterpret_cast<const uint4*>(x);
-    constexpr int U = 4;
-    for (int base = v0 + tid; base < v1; base += U * kThreads) {
-      uint4 buf[U];
+    for (int base = v0 + tid; base - tid < v1; base += 2 * kThreads) {
+      uint4 buf[2];
 #pragma unroll
-      for (int u = 0; u < U; ++u) {
-        int v = base + u * kThreads;
+      for (int u = 0; u < 2; ++u) {
+        const int v = base + u * kThreads;
         if (v < v1) buf[u] = __ldcs(xv + v);
       }
+      uint64_t k[EPT];
 #pragma unroll
-      for (int u = 0; u < U; ++u) {
-        int v = base + u * kThreads;
+      for (int u = 0; u < 2; ++u) {
+        const int v = base + u * kThreads;
+        const T* e = reinterpret_cast<const T*>(&buf[u]);
         if (v < v1) {
-          const T* e = reinterpret_cast<const T*>(&buf[u]);
           float vals[VE];
           float vmax = -INFINITY;
 #pragma unroll
@@ -246,46 +299,59 @@ topk_marginals_kernel(const T* __restrict__ logits, int64_t row_stride, int V, i
           }
           stats_raise(st, vmax * kLog2e);
 #pragma unroll
-          for (int i = 0; i < VE; ++i)
-            consume<KP, T>(vals[i], static_cast<uint32_t>(v * VE + i), st, lst);
+          for (int i = 0; i < VE; ++i) {
+            stats_add(st, vals[i] * kLog2e);
+            k[u * VE + i] = make_key(vals[i], static_cast<uint32_t>(v * VE + i));
+          }
+        } else {
+#pragma unroll
+          for (int i = 0; i < VE; ++i) k[u * VE + i] = 0;
         }
       }
+      merge_tile(k);
     }
     // tail elements past the last full vector go to the last chunk
-    if (chunk == chunks - 1) {
-      for (int i = nvec * VE + tid; i < V; i += kThreads) {
-        float xv1 = to_f32<T>(x[i]);
+    if (chunk == chunks - 1 && nvec * VE < V) {
+      uint64_t k[EPT];
+#pragma unroll
+      for (int i = 0; i < EPT; ++i) k[i] = 0;
+      const int i = nvec * VE + tid;   // fewer than VE tail elements
+      if (i < V) {
+        const float xv1 = to_f32<T>(x[i]);
         stats_raise(st, xv1 * kLog2e);
-        consume<KP, T>(xv1, static_cast<uint32_t>(i), st, lst);
+        stats_add(st, xv1 * kLog2e);
+        k[0] = make_key(xv1, static_cast<uint32_t>(i));
       }
+      merge_tile(k);
     }
   } else {
     const int per = (V + chunks - 1) / chunks;
     const int e0 = chunk * per;
     const int e1 = min(V, e0 + per);
-    for (int i = e0 + tid; i < e1; i += kThreads) {
-      float xv1 = to_f32<T>(x[i]);
-      stats_raise(st, xv1 * kLog2e);
-      consume<KP, T>(xv1, static_cast<uint32_t>(i), st, lst);
-    }
-  }
-
-  // ---- warp merge: KP rounds of a 64-bit warp maximum over list heads
-  for (int r = 0; r < KP; ++r) {
-    uint64_t best = warp_max_u64(lst[0]);
-    if (lane == 0) s_cand[warp * KP + r] = best;
-    if (best != 0 && lst[0] == best) {
+    for (int base = e0; base < e1; base += EPT * kThreads) {
+      uint64_t k[EPT];
 #pragma unroll
-      for (int i = 0; i < KP - 1; ++i) lst[i] = lst[i + 1];
-      lst[KP - 1] = 0;
+      for (int u = 0; u < EPT; ++u) {
+        const int i = base + u * kThreads + tid;
+        k[u] = 0;
+        if (i < e1) {
+          const float xv1 = to_f32<T>(x[i]);
+          stats_raise(st, xv1 * kLog2e);
+          stats_add(st, xv1 * kLog2e);
+          k[u] = make_key(xv1, static_cast<uint32_t>(i));
+        }
+      }
+      merge_tile(k);
     }
   }
+  if (lane < KP) s_cand[warp * KP + lane] = run;
   st = warp_stats(st);
   if (lane == 0) s_wstats[warp] = st;
   __syncthreads();
 
   if (warp == 0) {
-    warp_select_smem<KP>(s_cand, kWarps * KP, s_top, lane);
+    warp_top<KP>(s_cand, kWarps * KP, s_top, lane);
+    __syncwarp();
     Stats cs = s_wstats[0];
     for (int w = 1; w < kWarps; ++w) cs = stats_merge(cs, s_wstats[w]);
     if (chunks == 1) {
@@ -311,6 +377,15 @@ topk_marginals_kernel(const T* __restrict__ logits, int64_t row_stride, int V, i
   const int64_t rec0 = static_cast<int64_t>(row) * chunks;
   for (int i = tid; i < chunks * KP; i += kThreads) s_cand[i] = __ldcg(ws_keys + rec0 * KP + i);
   __syncthreads();
+  {
+    // each warp reduces a slice of at most 256 keys, then warp 0 the 8 results
+    const int n = chunks * KP, slice = (n + kWarps - 1) / kWarps;
+    const int lo = min(n, warp * slice), hi = min(n, lo + slice);
+    warp_top<KP>(s_cand + lo, hi - lo, s_part + warp * KP, lane);
+  }
+  __syncthreads();
+  if (warp == 0) warp_top<KP>(s_part, kWarps * KP, s_top, lane);
+  __syncthreads();
   if (warp == 0) {
     Stats cs{-INFINITY, 0.f, 0.f};
     for (int c = lane; c < chunks; c += 32) {
@@ -318,8 +393,6 @@ topk_marginals_kernel(const T* __restrict__ logits, int64_t row_stride, int V, i
       cs = stats_merge(cs, Stats{p.x, p.y, p.z});
     }
     cs = warp_stats(cs);
-    warp_select_smem<KP>(s_cand, chunks * KP, s_top, lane);
-    __syncwarp();
     write_row<KP>(row, K, s_top, cs, lane, ids, logp, lse, ent);
     if (lane == 0) tickets[row] = 0u;
   }
