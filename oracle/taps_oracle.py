@@ -24,6 +24,11 @@ notation, slowly and plainly:
                        tree attention (textbook masked softmax attention).
 * ``accept``           Sec. 4.1 and Limitations: greedy (temperature 0)
                        verification, the longest accepted root path.
+* ``target_greedy``    Limitations: at temperature 0 the target's choice at a
+                       node is the argmax of its verify logits.
+* ``compact_accepted_kv``  Sec. 4.1 (the loop alternates drafting and
+                       verification): the accepted path becomes committed
+                       context, so its K/V move to consecutive positions.
 
 Precision. Where the paper fixes no precision the oracle computes in float64
 (marginal statistics, scorer, attention). Reach and utility decide which nodes
@@ -47,6 +52,12 @@ Readings of the paper that this oracle encodes (the paper is silent there):
 7. Attention: scale 1/sqrt(D), contiguous GQA groups, a tree node sees the
    whole context plus its ancestors-or-self; tree node j's K/V sit at logical
    cache position ctx_len + j.
+8. Target greedy token: the first (lowest) vocabulary index attaining the
+   maximum logit; -0.0 and +0.0 are equal values.
+9. After acceptance, the K/V of accepted node path[i] (path[0] = root) moves
+   to logical position ctx_len + i; nothing else in the cache changes. The
+   node's K was computed at position id ctx_len + depth = ctx_len + i, so no
+   re-rotation is needed.
 """
 from __future__ import annotations
 
@@ -373,6 +384,50 @@ def accept(parent, token, n_nodes, target_tok, L):
         nodes[b, :len(path)] = path
         bonus[b] = int(target_tok[b, v])
     return accept_len, nodes, bonus
+
+
+def target_greedy(verify_logits, n_nodes):
+    """Target greedy token of every tree node (Limitations: temperature 0).
+
+    verify_logits [B, n_max, V]: the target's next-token logits after the
+    prefix ending at node i. Returns target_tok [B, n_max] int32: for i <
+    n_nodes[b] the lowest index whose logit equals the row maximum, else -1.
+    """
+    x = np.asarray(verify_logits, dtype=np.float64)
+    B, N, _ = x.shape
+    out = np.full((B, N), -1, np.int32)
+    for b in range(B):
+        for i in range(int(n_nodes[b])):
+            row = x[b, i]
+            top = row.max()
+            out[b, i] = int(np.flatnonzero(row == top)[0])
+    return out
+
+
+def compact_accepted_kv(k_cache, v_cache, block_table, ctx_len, accepted_nodes, accept_len,
+                        page=16):
+    """Move the accepted path's K/V to consecutive logical positions.
+
+    k_cache, v_cache: logical [num_pages, Hkv, page, D] caches of one layer.
+    Logical position t of request b is row t % page of page
+    block_table[b, t // page]. For i = 0 .. accept_len[b], the value at
+    position ctx_len[b] + accepted_nodes[b, i] (read before any write) is
+    written to position ctx_len[b] + i. Returns new arrays; inputs are unchanged.
+    """
+    k_new = np.array(k_cache, copy=True)
+    v_new = np.array(v_cache, copy=True)
+
+    def where(b, t):
+        return int(block_table[b, t // page]), t % page
+
+    for b in range(len(ctx_len)):
+        c = int(ctx_len[b])
+        for i in range(int(accept_len[b]) + 1):
+            sp, sr = where(b, c + int(accepted_nodes[b, i]))
+            dp, dr = where(b, c + i)
+            k_new[dp, :, dr, :] = k_cache[sp, :, sr, :]
+            v_new[dp, :, dr, :] = v_cache[sp, :, sr, :]
+    return k_new, v_new
 
 
 # ---------------------------------------------------------------------------

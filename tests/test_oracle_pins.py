@@ -582,3 +582,105 @@ def test_accept_chain_is_longest_prefix_match():
         alen, nodes, bonus = O.accept(parent, token, np.array([7]), tt, L)
         assert alen[0] == expect
         assert bonus[0] == y[0, expect]
+
+
+# ---------------------------------------------------------------------------
+# Target greedy token (temperature 0) and the accepted path's K/V compaction
+# ---------------------------------------------------------------------------
+
+def _first_max_python(row):
+    best = 0
+    for i in range(1, len(row)):
+        if float(row[i]) > float(row[best]):
+            best = i
+    return best
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_target_greedy_brute_force_with_ties(seed):
+    rng = np.random.default_rng(700 + seed)
+    B, N, V = 2, 5, 40
+    # few distinct values, so most rows have tied maxima
+    x = rng.integers(-3, 3, size=(B, N, V)).astype(np.float32)
+    x[0, 1] = -np.inf
+    x[0, 1, 17] = -0.0
+    x[0, 1, 23] = 0.0                      # -0.0 == +0.0: index 17 wins
+    x[1, 2] = -np.inf                      # all -inf: index 0
+    n_nodes = np.array([5, 3], np.int32)
+    t = O.target_greedy(x, n_nodes)
+    for b in range(B):
+        for i in range(N):
+            want = _first_max_python(x[b, i]) if i < n_nodes[b] else -1
+            assert t[b, i] == want, (b, i)
+    assert t[0, 1] == 17 and t[1, 2] == 0
+
+
+def test_target_greedy_planted_spike_gives_target_tokens():
+    """Verify logits whose row i peaks at y[depth(i)] reproduce the tree's target tokens."""
+    rng = np.random.default_rng(11)
+    L, K, V = 5, 3, 64
+    q = _random_qcond(rng, L, K)[None]
+    ids = np.stack([rng.permutation(V)[:K] for _ in range(L)]).astype(np.int32)[None]
+    s = O.select_subtree(q, ids, np.array([0]), np.array([0]), 1.0, 0.1, 0.0, 24)
+    y = rng.integers(0, V, size=(1, L + 1)).astype(np.int32)
+    tt = W.target_tokens_for_tree(y, s["depth"], s["n_nodes"])
+    x = rng.standard_normal((1, 24, V)).astype(np.float32)
+    n = int(s["n_nodes"][0])
+    for i in range(n):
+        x[0, i, tt[0, i]] = 50.0
+    got = O.target_greedy(x, s["n_nodes"])
+    assert (got[0, :n] == tt[0, :n]).all() and (got[0, n:] == -1).all()
+
+
+def _labelled_cache(num_pages, Hkv=2, D=4, page=16):
+    """Cache whose entry at (page p, head h, row r, dim d) encodes all four."""
+    p, h, r, d = np.meshgrid(np.arange(num_pages), np.arange(Hkv), np.arange(page),
+                             np.arange(D), indexing="ij")
+    return (p * 100000 + h * 10000 + r * 100 + d).astype(np.float64)
+
+
+def test_compact_chain_path_is_identity():
+    bt = np.array([[3, 0, 2, 1]], np.int32)
+    k = _labelled_cache(4)
+    v = -k
+    path = np.array([[0, 1, 2, 3, 4, 5]], np.int32)
+    kn, vn = O.compact_accepted_kv(k, v, bt, np.array([20]), path, np.array([5]))
+    assert (kn == k).all() and (vn == v).all()
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_compact_moves_each_accepted_row_and_nothing_else(seed):
+    rng = np.random.default_rng(900 + seed)
+    B, L, page = 3, 6, 16
+    ctx = np.array([5, 30, 16], np.int32)
+    n_tree = 40
+    need = (ctx + n_tree + page - 1) // page
+    perm = rng.permutation(int(need.sum()) + 2).astype(np.int32)
+    bt = np.full((B, int(need.max())), -1, np.int32)
+    o = 0
+    for b in range(B):
+        bt[b, :need[b]] = perm[o:o + need[b]]
+        o += int(need[b])
+    k = _labelled_cache(len(perm))
+    v = k + 0.5
+    alen = rng.integers(0, L + 1, size=B).astype(np.int32)
+    path = np.full((B, L + 1), -1, np.int32)
+    for b in range(B):
+        steps = np.sort(rng.choice(np.arange(1, n_tree), size=alen[b], replace=False))
+        path[b, :alen[b] + 1] = np.concatenate([[0], steps])
+    kn, vn = O.compact_accepted_kv(k, v, bt, ctx, path, alen)
+
+    def at(c, b, t):
+        return c[bt[b, t // page], :, t % page, :]
+
+    touched = set()
+    for b in range(B):
+        for i in range(alen[b] + 1):
+            dst, src = ctx[b] + i, ctx[b] + path[b, i]
+            assert (at(kn, b, dst) == at(k, b, src)).all()
+            assert (at(vn, b, dst) == at(v, b, src)).all()
+            touched.add((int(bt[b, dst // page]), dst % page))
+    for p in range(len(perm)):
+        for r in range(page):
+            if (p, r) not in touched:
+                assert (kn[p, :, r] == k[p, :, r]).all() and (vn[p, :, r] == v[p, :, r]).all()
