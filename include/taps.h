@@ -14,6 +14,14 @@
  *   taps_accept            Sec. 4.1 and Limitations (greedy, temperature 0,
  *                          lossless acceptance of the longest matching path)
  *
+ * and two steps that follow verification in the decoding loop:
+ *
+ *   taps_target_greedy_accept  Limitations (temperature 0: the target's
+ *                          choice is the argmax of its verify logits) fused
+ *                          with the acceptance walk of taps_accept
+ *   taps_compact_accepted_kv   Sec. 4.1 (drafting and verification
+ *                          alternate: the accepted path becomes context)
+ *
  * Conventions shared by every call:
  *  - Array arguments are DEVICE pointers owned by the caller. The library never
  *    allocates, frees or synchronises; every call is asynchronous on `stream`
@@ -63,6 +71,7 @@ enum { TAPS_DEVFAULT_PAGE = 1, TAPS_DEVFAULT_TIMEOUT = 2 };
 #define TAPS_MAX_NODES 512
 #define TAPS_MAX_EMB 32
 #define TAPS_MAX_HIDDEN 64
+#define TAPS_MAX_LAYERS 128
 
 const char* taps_status_string(int status);
 int taps_version(void);
@@ -274,6 +283,63 @@ int taps_unpack_kv_pages(const void* src, void* dst, int64_t num_pages, int Hkv,
 int taps_accept(const int32_t* parent, const int32_t* token, const int32_t* n_nodes,
                 const int32_t* target_tok, int B, int n_max, int L,
                 int32_t* accept_len, int32_t* accepted_nodes, int32_t* bonus_tok, void* stream);
+
+/* ------------------------------------------------------------------------
+ * taps_target_greedy_accept - the target's greedy token at every tree node,
+ * fused with the acceptance walk. At temperature 0 (Limitations) the target
+ * accepts a draft token iff it equals the argmax of the target's logits after
+ * the prefix ending at the node's parent; Sec. 4.1 then keeps the longest
+ * root path of accepted tokens.
+ *
+ * verify_logits [B, n_max, V] of dtype TAPS_F32 or TAPS_BF16: the target's
+ *          next-token logits after the prefix ending at tree node i; row
+ *          (b, i) starts at element (b * n_max + i) * row_stride. Only rows
+ *          i < n_nodes[b] are read.
+ * parent, token, n_nodes as written by taps_select_subtree.
+ * target_tok [B, n_max] int32, out: the lowest vocabulary index attaining the
+ *          row's maximum (-0.0 equals +0.0) for i < n_nodes[b], else -1.
+ * accept_len, accepted_nodes, bonus_tok: out, exactly as taps_accept computes
+ *          them from target_tok.
+ * ws       workspace of taps_target_greedy_accept_workspace_bytes(B, n_max),
+ *          zero-filled before the first call; every call leaves it at zero.
+ * Limits: n_max <= 512, L <= 31, row_stride >= V. Logits must not be NaN.
+ * ---------------------------------------------------------------------- */
+size_t taps_target_greedy_accept_workspace_bytes(int B, int n_max);
+int taps_target_greedy_accept(const void* verify_logits, int dtype, int64_t row_stride,
+                              int B, int n_max, int V, const int32_t* parent,
+                              const int32_t* token, const int32_t* n_nodes, int L,
+                              int32_t* target_tok, int32_t* accept_len, int32_t* accepted_nodes,
+                              int32_t* bonus_tok, void* ws, size_t ws_bytes, void* stream);
+
+/* ------------------------------------------------------------------------
+ * taps_compact_accepted_kv - commit the accepted path to the KV cache. The
+ * decoding loop alternates drafting and verification (Sec. 4.1): after
+ * acceptance the accepted tokens are context for the next round, so for
+ * i = 0 .. accept_len[b] the K and V at logical position
+ * ctx_len[b] + accepted_nodes[b, i] (where verification left tree node
+ * accepted_nodes[b, i]) move to position ctx_len[b] + i, in every layer.
+ * All reads of a (layer, request, head) finish before its writes; no other
+ * position changes. Keys need no re-rotation: the node at path index i has
+ * depth i, and its key was rotated at position id ctx_len[b] + i.
+ *
+ * k_layers, v_layers  HOST arrays of num_layers DEVICE pointers, one K and
+ *          one V cache per layer, each [num_pages, Hkv, 16, D] bf16 in the
+ *          TAPS page layout (16-byte aligned), updated in place.
+ * block_table [B, max_pages], ctx_len [B] as for taps_tree_verify_attn; the
+ *          pages holding positions >= ctx_len[b] must belong to request b
+ *          alone.
+ * accepted_nodes [B, L + 1], accept_len [B] as written by taps_accept.
+ * status   device int32, nullable: TAPS_DEVFAULT_PAGE is ORed in when a
+ *          position falls outside the block table or a page id outside
+ *          [0, num_pages); that move is skipped.
+ * Limits: num_layers <= TAPS_MAX_LAYERS, L <= 31, page_size == 16,
+ *         D in {64, 128}.
+ * ---------------------------------------------------------------------- */
+int taps_compact_accepted_kv(void* const* k_layers, void* const* v_layers, int num_layers,
+                             int64_t num_pages, const int32_t* block_table, int max_pages,
+                             const int32_t* ctx_len, const int32_t* accepted_nodes,
+                             const int32_t* accept_len, int B, int L, int Hkv, int D,
+                             int page_size, int32_t* status, void* stream);
 
 #ifdef __cplusplus
 }

@@ -346,3 +346,81 @@ def taps_unpack_kv_pages(cache: torch.Tensor, out: torch.Tensor | None = None, s
                                   _stream(stream, cache.device))
     _check("taps_unpack_kv_pages", st)
     return out
+
+
+# ---------------------------------------------------------------------------
+# steps after verification: target greedy tokens + acceptance, K/V commit
+# ---------------------------------------------------------------------------
+
+lib.taps_target_greedy_accept_workspace_bytes.argtypes = [_I, _I]
+lib.taps_target_greedy_accept_workspace_bytes.restype = _SZ
+lib.taps_target_greedy_accept.argtypes = [_P, _I, _I64, _I, _I, _I, _P, _P, _P, _I, _P, _P, _P,
+                                          _P, _P, _SZ, _P]
+lib.taps_target_greedy_accept.restype = _I
+lib.taps_compact_accepted_kv.argtypes = [ctypes.POINTER(_P), ctypes.POINTER(_P), _I, _I64, _P,
+                                         _I, _P, _P, _P, _I, _I, _I, _I, _I, _P, _P]
+lib.taps_compact_accepted_kv.restype = _I
+
+
+def target_greedy_accept_workspace_bytes(B, n_max) -> int:
+    return int(lib.taps_target_greedy_accept_workspace_bytes(B, n_max))
+
+
+def taps_target_greedy_accept(verify_logits: torch.Tensor, parent, token, n_nodes, L,
+                              out=None, ws=None, stream=None):
+    """Target greedy token per tree node fused with acceptance: returns
+    (target_tok [B, n_max], accept_len [B], accepted_nodes [B, L+1], bonus_tok [B])."""
+    if verify_logits.dtype not in (torch.float32, torch.bfloat16) or not verify_logits.is_cuda:
+        raise TypeError("verify_logits must be a CUDA float32 or bfloat16 tensor")
+    B, n_max, V = verify_logits.shape
+    if verify_logits.stride(2) != 1 or verify_logits.stride(0) != n_max * verify_logits.stride(1):
+        raise ValueError("verify_logits rows must be unit-stride with a uniform row stride")
+    _need(parent, torch.int32, (B, n_max), "parent")
+    _need(token, torch.int32, (B, n_max), "token")
+    _need(n_nodes, torch.int32, (B,), "n_nodes")
+    dev = verify_logits.device
+    if out is None:
+        out = (torch.empty((B, n_max), dtype=torch.int32, device=dev),
+               torch.empty(B, dtype=torch.int32, device=dev),
+               torch.empty((B, L + 1), dtype=torch.int32, device=dev),
+               torch.empty(B, dtype=torch.int32, device=dev))
+    tt, alen, nodes, bonus = out
+    _need(tt, torch.int32, (B, n_max), "target_tok")
+    _need(alen, torch.int32, (B,), "accept_len")
+    _need(nodes, torch.int32, (B, L + 1), "accepted_nodes")
+    _need(bonus, torch.int32, (B,), "bonus_tok")
+    nb = target_greedy_accept_workspace_bytes(B, n_max)
+    if ws is None:
+        ws = workspace(nb, dev, "target", stream)
+    dtype = TAPS_F32 if verify_logits.dtype == torch.float32 else TAPS_BF16
+    st = lib.taps_target_greedy_accept(_ptr(verify_logits), dtype, verify_logits.stride(1), B,
+                                       n_max, V, _ptr(parent), _ptr(token), _ptr(n_nodes), L,
+                                       _ptr(tt), _ptr(alen), _ptr(nodes), _ptr(bonus), _ptr(ws),
+                                       nb, _stream(stream, dev))
+    _check("taps_target_greedy_accept", st)
+    return tt, alen, nodes, bonus
+
+
+def taps_compact_accepted_kv(k_layers, v_layers, block_table, ctx_len, accepted_nodes,
+                             accept_len, status=None, stream=None):
+    """Move each layer's accepted-path K/V to consecutive positions after
+    ctx_len (in place). k_layers / v_layers: lists of TAPS-layout caches."""
+    if len(k_layers) != len(v_layers) or not k_layers:
+        raise ValueError("need one K and one V cache per layer")
+    num_pages, Hkv, P, D = k_layers[0].shape
+    for t in list(k_layers) + list(v_layers):
+        _need(t, torch.bfloat16, (num_pages, Hkv, P, D), "cache")
+    B, max_pages = block_table.shape
+    _need(block_table, torch.int32, (B, max_pages), "block_table")
+    _need(ctx_len, torch.int32, (B,), "ctx_len")
+    L = accepted_nodes.shape[1] - 1
+    _need(accepted_nodes, torch.int32, (B, L + 1), "accepted_nodes")
+    _need(accept_len, torch.int32, (B,), "accept_len")
+    n = len(k_layers)
+    kp = (_P * n)(*[t.data_ptr() for t in k_layers])
+    vp = (_P * n)(*[t.data_ptr() for t in v_layers])
+    dev = k_layers[0].device
+    st = lib.taps_compact_accepted_kv(kp, vp, n, num_pages, _ptr(block_table), max_pages,
+                                      _ptr(ctx_len), _ptr(accepted_nodes), _ptr(accept_len), B,
+                                      L, Hkv, D, P, _ptr(status), _stream(stream, dev))
+    _check("taps_compact_accepted_kv", st)

@@ -117,3 +117,43 @@ def test_attention_rejects_bad_arguments(lib):
     assert call(Hq=80, Hkv=8) == 2                                   # group 10 > 8
     assert call(Hq=24, Hkv=8) == 2                                   # group 3
     assert call(ctx=65536 - 63) == 2                                 # ctx + n_max > 65536
+
+
+def test_target_greedy_accept_rejects_bad_arguments(lib):
+    tb = _b()
+    f = tb.lib.taps_target_greedy_accept
+    WS = ctypes.c_void_p(0x10000)      # 256-byte aligned, never dereferenced
+    nb = tb.target_greedy_accept_workspace_bytes(2, 64)
+    assert nb >= 2 * 64 * 8 and tb.target_greedy_accept_workspace_bytes(0, 64) == 0
+
+    def call(x=FAKE, dtype=1, stride=1000, B=2, n=64, V=1000, L=16, ws=WS, wsb=nb):
+        return f(x, dtype, stride, B, n, V, FAKE, FAKE, FAKE, L, FAKE, FAKE, FAKE, FAKE, ws, wsb,
+                 None)
+    assert call(x=None) == 1
+    assert call(dtype=7) == 1
+    assert call(stride=999) == 1
+    assert call(V=0) == 1
+    assert call(n=600) == 2
+    assert call(L=32) == 2
+    assert call(ws=None) == 3
+    assert call(wsb=nb - 1) == 3
+    assert call(ws=ctypes.c_void_p(0x10010)) == 3                     # not 256-byte aligned
+
+
+def test_compact_accepted_kv_rejects_bad_arguments(lib):
+    tb = _b()
+    f = tb.lib.taps_compact_accepted_kv
+    ptrs = (ctypes.c_void_p * 2)(0x1000, 0x2000)
+
+    def call(k=ptrs, v=ptrs, layers=2, pages=10, L=16, Hkv=8, D=128, P=16, bt=FAKE):
+        return f(k, v, layers, pages, bt, 4, FAKE, FAKE, FAKE, 1, L, Hkv, D, P, None, None)
+    assert call(k=None) == 1
+    assert call(bt=None) == 1
+    assert call(layers=0) == 1
+    assert call(pages=0) == 1
+    assert call(layers=129) == 2
+    assert call(L=32) == 2
+    assert call(D=96) == 2
+    assert call(P=32) == 2
+    bad = (ctypes.c_void_p * 2)(0x1000, 0x2008)                        # not 16-byte aligned
+    assert call(v=bad) == 1

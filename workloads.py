@@ -297,3 +297,19 @@ def make_q_torch(cfg: RoundConfig, B: int, n_max: int, layer: int, device):
     g.manual_seed(SEED_BASE * 1000 + 50000 + cfg.config_id * 100 + layer)
     return torch.randn((B, n_max, cfg.Hq, cfg.D), generator=g, device=device,
                        dtype=torch.float32).to(torch.bfloat16)
+
+
+def make_verify_logits_torch(cfg: RoundConfig, target_tok, device, seed_offset: int = 0):
+    """Target verify logits [B, n_max, V] bf16 on the device, drawn N(0, 4), with
+    the value 24 (12 standard deviations) planted at target_tok[b, i] for every
+    row whose token is >= 0, so the row's greedy token is the stand-in
+    target's token."""
+    import torch
+    g = torch.Generator(device=device)
+    g.manual_seed(SEED_BASE * 1000 + 90000 + cfg.config_id * 100 + seed_offset)
+    B, N = target_tok.shape
+    x = torch.randn((B, N, cfg.V), generator=g, device=device, dtype=torch.float32) * 2.0
+    tt = target_tok.to(device=device, dtype=torch.int64)
+    b, i = torch.nonzero(tt >= 0, as_tuple=True)
+    x[b, i, tt[b, i]] = 24.0
+    return x.to(torch.bfloat16)
