@@ -57,10 +57,20 @@ def load_peaks():
         return FALLBACK_HBM_GBS, FALLBACK_BF16_TFLOPS, "fallback"
 
 
-def workload_config(name, n_max, layers):
+def workload_config(name, n_max=None, layers=None):
     import workloads as W
     cfg = W.CONFIGS[name]
-    return cfg.with_(n_max=n_max, layers=layers)
+    return cfg.with_(n_max=cfg.n_max if n_max is None else n_max,
+                     layers=cfg.layers if layers is None else layers)
+
+
+SHAPE_NAMES = {"qwen3_8b": "Qwen3-8B", "qwen3_4b": "Qwen3-4B", "llama31_8b": "LLaMA-3.1-8B",
+               "batched": "Qwen3-8B batch-32", "long": "Qwen3-8B long-context", "tiny": "tiny"}
+
+
+def metric_name(workload):
+    return (f"TAPS rounds/sec (select+tree verify) at {SHAPE_NAMES.get(workload, workload)} "
+            "shape, 1 GB300; % HBM roofline")
 
 
 def attn_bytes_flops(cfg, ctx, n_nodes, depth):
@@ -173,10 +183,11 @@ def cpu_child(args):
 
 
 def run_cpu_baseline(args, steps, warmup, sample_layers):
+    cfg = workload_config(args.workload, args.n_max, args.layers)
     env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1",
                CUDA_VISIBLE_DEVICES="")
     cmd = [sys.executable, os.path.abspath(__file__), "--cpu-child", "--workload", args.workload,
-           "--n-max", str(args.n_max), "--layers", str(args.layers), "--steps", str(steps),
+           "--n-max", str(cfg.n_max), "--layers", str(cfg.layers), "--steps", str(steps),
            "--warmup", str(warmup), "--sample-layers", str(sample_layers)]
     r = subprocess.run(cmd, env=env, capture_output=True, text=True)
     if r.returncode != 0:
@@ -502,19 +513,23 @@ def run_ours(args):
                 "tensor_frac": round(achieved_tf / bf16, 4)}
 
     launches = args.steps * (r.launches_per_select + cfg.layers * r.launches_per_layer + 1)
+    kv_bytes = sum(kc.numel() * kc.element_size() + vc.numel() * vc.element_size()
+                   for (_, kc, vc, _) in layers)
     line = {
-        "metric": "TAPS rounds/sec (select+tree verify) at Qwen3-8B shape, 1 GB300; % HBM roofline",
+        "metric": metric_name(args.workload),
         "value": round(world * args.steps / (elapsed_ms / 1e3), 2),
         "unit": "rounds/s",
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": round(elapsed_ms / args.steps, 4),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
-        "data": "synthetic (seeded; shapes of the Qwen3-8B round, no weights or datasets)",
+        "data": f"synthetic (seeded; shapes of the {SHAPE_NAMES.get(args.workload, args.workload)} "
+                "round, no weights or datasets)",
         "config": {"workload": f"{cfg.name}: B={cfg.B} L={cfg.L} V={cfg.V} K={cfg.K} "
                                f"n_max={cfg.n_max} layers={cfg.layers} Hq={cfg.Hq} Hkv={cfg.Hkv} "
                                f"D={cfg.D} ctx={cfg.ctx} page={cfg.page}",
                    "global_batch": cfg.B, "seq_len": int(ctx_h.max()), "parallelism": "replicas",
-                   "l2": "inputs larger than L2: 36 distinct KV layers, 0.6 GB per step",
+                   "l2": f"inputs larger than L2: {cfg.layers} distinct KV layers, "
+                         f"{kv_bytes / 1e9:.1f} GB per step",
                    "n_nodes": int(sel_h["n_nodes"][0]),
                    "select_plus_one_layer_round_us": round(one_layer_us, 2),
                    "attention_stage_us_per_round": round(attn_ms * 1e3, 2)},
@@ -550,11 +565,12 @@ def run_reference(args):
     value = args.steps / total
     line = {
         "impl": "reference",
-        "metric": "TAPS rounds/sec (select+tree verify) at Qwen3-8B shape, 1 GB300; % HBM roofline",
+        "metric": metric_name(args.workload),
         "value": round(value, 5), "unit": "rounds/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(total / args.steps * 1e3, 2),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-        "data": "synthetic (seeded; shapes of the Qwen3-8B round, no weights or datasets)",
+        "data": f"synthetic (seeded; shapes of the {SHAPE_NAMES.get(args.workload, args.workload)} "
+                "round, no weights or datasets)",
         "config": {"workload": f"{cfg.name}: B={cfg.B} L={cfg.L} V={cfg.V} K={cfg.K} "
                                f"n_max={cfg.n_max} layers={cfg.layers} Hq={cfg.Hq} Hkv={cfg.Hkv} "
                                f"D={cfg.D} ctx={cfg.ctx} page={cfg.page}",
@@ -575,8 +591,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="qwen3_8b")
-    ap.add_argument("--n-max", type=int, default=64)
-    ap.add_argument("--layers", type=int, default=36)
+    ap.add_argument("--n-max", type=int, default=None, help="node budget (default: workload's)")
+    ap.add_argument("--layers", type=int, default=None, help="layers (default: workload's)")
     ap.add_argument("--sample-layers", type=int, default=3)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")

@@ -2,7 +2,10 @@
 
 Sequencing only: the six stages run in the order of Sec. 4.1 (top-K
 marginals -> scoring -> selection -> mask -> per-layer tree verification ->
-acceptance), each as one call into libtaps.so on the caller's stream. All
+acceptance), each as one call into libtaps.so on the caller's stream. With
+the target's verify logits at hand, acceptance can instead take the greedy
+token of every node from them (accept_greedy), and commit_kv moves the
+accepted path's K/V into place for the next round. All
 outputs and workspaces are allocated once here, so a round can be captured
 in a CUDA graph and replayed.
 """
@@ -38,6 +41,9 @@ class TapsRound:
         self.accepted_nodes = torch.empty((B, L + 1), dtype=i32, device=dev)
         self.bonus_tok = torch.empty(B, dtype=i32, device=dev)
         self.status = torch.zeros(1, dtype=i32, device=dev)
+        self.target_tok = torch.empty((B, n_max), dtype=i32, device=dev)
+        nb = tb.target_greedy_accept_workspace_bytes(B, n_max)
+        self.ws_target = torch.zeros(max(nb, 1), dtype=torch.uint8, device=dev)
         nb = tb.topk_marginals_workspace_bytes(B, L, V, K)
         self.ws_topk = torch.zeros(max(nb, 1), dtype=torch.uint8, device=dev)
         nb = tb.tree_verify_attn_workspace_bytes(B, n_max, Hq, Hkv, D, max_ctx)
@@ -71,6 +77,23 @@ class TapsRound:
         tb.taps_accept(self.sel["parent"], self.sel["token"], self.sel["n_nodes"], target_tok,
                        self.L, out=(self.accept_len, self.accepted_nodes, self.bonus_tok),
                        stream=stream)
+
+    def accept_greedy(self, verify_logits, stream=None):
+        """Target greedy token of every node (argmax of its verify logits
+        [B, n_max, V]) fused with acceptance; fills target_tok as well."""
+        tb.taps_target_greedy_accept(verify_logits, self.sel["parent"], self.sel["token"],
+                                     self.sel["n_nodes"], self.L,
+                                     out=(self.target_tok, self.accept_len, self.accepted_nodes,
+                                          self.bonus_tok),
+                                     ws=self.ws_target, stream=stream)
+
+    def commit_kv(self, k_layers, v_layers, block_table, ctx_len, stream=None):
+        """Move the accepted path's K/V to positions ctx_len .. ctx_len +
+        accept_len in every layer; the caller then advances ctx_len by
+        accept_len + 1."""
+        tb.taps_compact_accepted_kv(k_layers, v_layers, block_table, ctx_len,
+                                    self.accepted_nodes, self.accept_len, status=self.status,
+                                    stream=stream)
 
     def run(self, logits, root_tok, ctx_len, layers, outs, target_tok, stream=None):
         """layers: list of (q, k_cache, v_cache, block_table); outs: one output per layer."""

@@ -61,7 +61,7 @@ def _check_topk(taps, x, K, dtype=torch.float32, x_dev=None):
     assert np.all(np.abs(host(logp) - r_logp) <= 1e-5 * scale)
 
 
-@pytest.mark.parametrize("name", ["tiny", "qwen3_4b", "qwen3_8b", "long"])
+@pytest.mark.parametrize("name", ["tiny", "qwen3_4b", "qwen3_8b", "long", "llama31_8b"])
 def test_topk_configs(taps, name):
     cfg = W.CONFIGS[name]
     B = min(cfg.B, 2)
@@ -117,7 +117,7 @@ def _stage1_inputs(cfg, B=None):
 
 @pytest.mark.parametrize("name,kind", [("tiny", "mlp"), ("tiny", "marginal"),
                                        ("qwen3_8b", "mlp"), ("long", "mlp"),
-                                       ("qwen3_8b", "marginal")])
+                                       ("qwen3_8b", "marginal"), ("llama31_8b", "mlp")])
 def test_score_parity(taps, name, kind):
     cfg = W.CONFIGS[name]
     x, ids, logp, ent, root = _stage1_inputs(cfg, B=min(cfg.B, 2))
@@ -150,6 +150,7 @@ def _check_select(taps, q, ids, root, ctx, l1, l2, tau, n_max):
 
 @pytest.mark.parametrize("name,n_max", [("tiny", 16), ("qwen3_8b", 32), ("qwen3_8b", 64),
                                         ("qwen3_8b", 128), ("qwen3_8b", 256), ("long", 256),
+                                        ("llama31_8b", 64),
                                         ("qwen3_4b", 512)])
 def test_select_parity(taps, name, n_max):
     cfg = W.CONFIGS[name]
@@ -355,7 +356,8 @@ def test_attention_ragged_batch_sampled(taps):
     _sampled_check(q, kc, vc, bt, ctx, nn, mask, out, np.random.default_rng(3), per_req=8)
 
 
-@pytest.mark.parametrize("name,n", [("qwen3_8b", 64), ("qwen3_8b", 256), ("qwen3_4b", 64)])
+@pytest.mark.parametrize("name,n", [("qwen3_8b", 64), ("qwen3_8b", 256), ("qwen3_4b", 64),
+                                    ("llama31_8b", 64)])
 def test_attention_full_size_sampled(taps, name, n):
     cfg = W.CONFIGS[name]
     ctx = W.make_ctx_lens(cfg)
@@ -473,7 +475,8 @@ def _near_tie_valid(tree, q_ref, ids, L, K, lambda1, lambda2, rtol=1e-5):
     return front_max <= sel_min * (1 + rtol)
 
 
-@pytest.mark.parametrize("name,n_max", [("tiny", 16), ("qwen3_8b", 64), ("qwen3_8b", 256)])
+@pytest.mark.parametrize("name,n_max", [("tiny", 16), ("qwen3_8b", 64), ("qwen3_8b", 256),
+                                        ("llama31_8b", 64)])
 def test_round_end_to_end(taps, name, n_max):
     cfg = W.CONFIGS[name]
     x = W.make_logits(cfg)

@@ -85,6 +85,11 @@ CONFIGS = {
     "long": RoundConfig("long", B=8, L=16, V=151936, K=16, n_max=256, logits_kind="bimodal",
                         logits_dtype="bf16", layers=36, Hq=32, Hkv=8, D=128, ctx=32768,
                         config_id=4),
+    # LLaMA-3.1-8B-Instruct target: draft block 10, vocabulary 128256, 32 layers
+    # of 32 query / 8 KV heads of dimension 128
+    "llama31_8b": RoundConfig("llama31_8b", B=1, L=10, V=128256, K=8, n_max=64,
+                              logits_kind="zipf_temp", logits_dtype="bf16", layers=32, Hq=32,
+                              Hkv=8, D=128, ctx=4096, config_id=5),
 }
 
 
