@@ -45,6 +45,7 @@ Readings of the paper that this oracle encodes (the paper is silent there):
    over [E_tok[parent], E_tok[child], E_dep[depth], logp(child), H(depth)],
    plus w_lp * logp(child). Kind ``marginal`` is the paper's ablation that
    ranks by the drafter's marginal confidence: logit = logp(child).
+   Kind ``marginal_product`` (DDTree-style) uses q = exp(logp(child)) as is.
 4. Utility threshold is strict (utility > tau).
 5. Total order used by argmax: utility desc, depth asc, token id asc, parent's
    position in the greedy order asc. Top-K ties: logit desc, token id asc.
@@ -58,6 +59,11 @@ Readings of the paper that this oracle encodes (the paper is silent there):
    to logical position ctx_len + i; nothing else in the cache changes. The
    node's K was computed at position id ctx_len + depth = ctx_len + i, so no
    re-rotation is needed.
+10. Ablation presets (Sec. 5.3): "no target-aware pruning" keeps the scorer
+   and selects without the cost term or threshold (lambda2 = 0, tau = 0);
+   with lambda2 = 0 the utility is reach / lambda1, so Algorithm 1 fills the
+   budget in descending reach. DDTree-style selection is that rule over
+   marginal path probabilities.
 """
 from __future__ import annotations
 
@@ -128,6 +134,10 @@ def score_qcond(root_tok, ids, logp, entropy, kind: str = "mlp", weights: dict |
     Parent i is slot i of position d-1, or the root when d == 0 (row i = 0;
     rows i >= 1 at d == 0 are zero). For each parent the scorer logits of its K
     children are normalised with a sibling-wise softmax (Eq. 1, Algorithm 1).
+    Kind ``marginal_product`` is the DDTree-style ranking the paper contrasts
+    TAPS with (Sec. 3.1, Limitation 1: nodes chosen by the drafter's marginal
+    probabilities): no scorer and no renormalisation, q = exp(logp(child)), so
+    the reach of a node is the product of its path's marginal probabilities.
     Computed in float64, returned as float32.
     """
     B, L, K = ids.shape
@@ -138,13 +148,16 @@ def score_qcond(root_tok, ids, logp, entropy, kind: str = "mlp", weights: dict |
             for i, ptok in enumerate(parents):
                 ell = np.empty(K, np.float64)
                 for j in range(K):
-                    if kind == "marginal":
+                    if kind in ("marginal", "marginal_product"):
                         ell[j] = float(logp[b, d, j])
                     else:
                         ell[j] = edge_logit_mlp(weights, ptok, int(ids[b, d, j]), d + 1,
                                                 float(logp[b, d, j]), float(entropy[b, d]))
-                e = np.exp(ell - ell.max())
-                q[b, d, i] = e / e.sum()
+                if kind == "marginal_product":
+                    q[b, d, i] = np.exp(ell)
+                else:
+                    e = np.exp(ell - ell.max())
+                    q[b, d, i] = e / e.sum()
     return q.astype(F32)
 
 

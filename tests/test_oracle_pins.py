@@ -684,3 +684,77 @@ def test_compact_moves_each_accepted_row_and_nothing_else(seed):
         for r in range(page):
             if (p, r) not in touched:
                 assert (kn[p, :, r] == k[p, :, r]).all() and (vn[p, :, r] == v[p, :, r]).all()
+
+
+# ---------------------------------------------------------------------------
+# Ablation presets (Sec. 5.3) and the DDTree-style marginal ranking (Sec. 3.1)
+# ---------------------------------------------------------------------------
+
+def _all_slot_paths(L, K):
+    paths = [()]
+    for d in range(L):
+        paths += [p + (j,) for p in paths if len(p) == d for j in range(K)]
+    return paths
+
+
+def _selected_slot_paths(s, b=0):
+    n = int(s["n_nodes"][b])
+    paths = {0: ()}
+    for i in range(1, n):
+        paths[i] = paths[int(s["parent"][b, i])] + (int(s["slot"][b, i]),)
+    return set(paths.values())
+
+
+def _top_n(paths, score, n):
+    ranked = sorted(paths, key=lambda p: -score(p))
+    # the cut must not fall on a near-tie, or float32 rounding could decide it
+    if len(ranked) > n:
+        a, b = score(ranked[n - 1]), score(ranked[n])
+        assert a > b * (1 + 1e-4), "seed gives a near-tie at the budget cut"
+    return set(ranked[:n])
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_budget_fill_is_top_n_by_reach(seed):
+    """lambda2 = 0, tau = 0: the selected set is the n_max trie nodes of
+    largest reach (reach only falls along a path, so that set is prefix-closed)."""
+    rng = np.random.default_rng(1100 + seed)
+    L, K, n_max = 4, 3, 15
+    q = _random_qcond(rng, L, K)
+    ids = np.stack([rng.permutation(20)[:K] for _ in range(L)]).astype(np.int32)
+    s = O.select_subtree(q[None], ids[None], np.array([0]), np.array([0]), 1.0, 0.0, 0.0, n_max)
+    assert int(s["n_nodes"][0]) == n_max                       # the budget is filled
+
+    def reach(p):                                               # float64 product along p
+        r = 1.0
+        for d, j in enumerate(p):
+            r *= float(q[d, 0 if d == 0 else p[d - 1], j])
+        return r
+
+    assert _selected_slot_paths(s) == _top_n(_all_slot_paths(L, K), reach, n_max)
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_ddtree_mode_is_top_n_by_marginal_path_probability(seed):
+    B, L, K, V = 1, 4, 3, 30
+    x, ids, logp, ent, root = _tiny_inputs(B=B, L=L, K=K, V=V, seed=1200 + seed)
+    q = O.score_qcond(root, ids, logp, ent, "marginal_product")
+    # closed form: each parent's row is the children's full-vocabulary marginals
+    z = np.asarray(x, np.float64)
+    p_full = np.exp(z - z.max(-1, keepdims=True))
+    p_full /= p_full.sum(-1, keepdims=True)
+    marg = np.take_along_axis(p_full[0], ids[0].astype(np.int64), axis=-1)     # [L, K]
+    for d in range(L):
+        for i in range(1 if d == 0 else K):
+            np.testing.assert_allclose(q[0, d, i], marg[d], rtol=1e-6)
+        assert q[0, d, 0].sum() <= 1.0 + 1e-6
+    n_max = 12
+    s = O.select_subtree(q, ids, root, np.array([0]), 1.0, 0.0, 0.0, n_max)
+
+    def path_prob(p):
+        r = 1.0
+        for d, j in enumerate(p):
+            r *= marg[d, j]
+        return r
+
+    assert _selected_slot_paths(s) == _top_n(_all_slot_paths(L, K), path_prob, n_max)
