@@ -57,11 +57,19 @@ def load_peaks():
         return FALLBACK_HBM_GBS, FALLBACK_BF16_TFLOPS, "fallback"
 
 
-def workload_config(name, n_max=None, layers=None):
+# scorer kind and (lambda2, tau) overrides of each selection preset; the
+# library's TapsRound takes the same presets by name
+MODE_PARAMS = {"taps": ("mlp", None), "no_scorer": ("marginal", None),
+               "budget_fill": ("mlp", (0.0, 0.0)), "ddtree": ("marginal_product", (0.0, 0.0))}
+
+
+def workload_config(name, n_max=None, layers=None, mode="taps"):
     import workloads as W
     cfg = W.CONFIGS[name]
-    return cfg.with_(n_max=cfg.n_max if n_max is None else n_max,
-                     layers=cfg.layers if layers is None else layers)
+    cfg = cfg.with_(n_max=cfg.n_max if n_max is None else n_max,
+                    layers=cfg.layers if layers is None else layers)
+    over = MODE_PARAMS[mode][1]
+    return cfg if over is None else cfg.with_(lambda2=over[0], tau=over[1])
 
 
 SHAPE_NAMES = {"qwen3_8b": "Qwen3-8B", "qwen3_4b": "Qwen3-4B", "llama31_8b": "LLaMA-3.1-8B",
@@ -133,14 +141,14 @@ class ClockSampler:
 # CPU baseline: the oracle as it stands, on a bounded sample of the workload
 # ---------------------------------------------------------------------------
 
-def oracle_step(cfg, inp, sample_layers):
+def oracle_step(cfg, inp, sample_layers, kind="mlp"):
     """One oracle round: stages 1-4 and 6 on the whole batch, stage 5 on
     ``sample_layers`` of the cfg.layers layers; returns seconds scaled to the
     full round."""
     from oracle import taps_oracle as O
     t0 = time.perf_counter()
     ids, logp, lse, ent = O.topk_marginals(inp["logits"], cfg.K)
-    q = O.score_qcond(inp["root"], ids, logp, ent, "mlp", inp["w"])
+    q = O.score_qcond(inp["root"], ids, logp, ent, kind, inp["w"])
     sel = O.select_subtree(q, ids, inp["root"], inp["ctx"], cfg.lambda1, cfg.lambda2, cfg.tau,
                            cfg.n_max)
     mask = O.build_tree_mask(sel["parent"], sel["n_nodes"], cfg.n_max)
@@ -169,24 +177,26 @@ def oracle_inputs(cfg):
 
 def cpu_child(args):
     """Runs in a fresh single-threaded process: prints the oracle timing JSON."""
-    cfg = workload_config(args.workload, args.n_max, args.layers)
+    cfg = workload_config(args.workload, args.n_max, args.layers, args.mode)
+    kind = MODE_PARAMS[args.mode][0]
     inp = oracle_inputs(cfg)
     steps, warm = args.steps, args.warmup
     for _ in range(warm):
-        oracle_step(cfg, inp, args.sample_layers)
+        oracle_step(cfg, inp, args.sample_layers, kind)
     scaled, wall = [], []
     for _ in range(steps):
-        s, w = oracle_step(cfg, inp, args.sample_layers)
+        s, w = oracle_step(cfg, inp, args.sample_layers, kind)
         scaled.append(s)
         wall.append(w)
     print(json.dumps({"scaled_s": scaled, "wall_s": wall}))
 
 
 def run_cpu_baseline(args, steps, warmup, sample_layers):
-    cfg = workload_config(args.workload, args.n_max, args.layers)
+    cfg = workload_config(args.workload, args.n_max, args.layers, args.mode)
     env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1",
                CUDA_VISIBLE_DEVICES="")
     cmd = [sys.executable, os.path.abspath(__file__), "--cpu-child", "--workload", args.workload,
+           "--mode", args.mode,
            "--n-max", str(cfg.n_max), "--layers", str(cfg.layers), "--steps", str(steps),
            "--warmup", str(warmup), "--sample-layers", str(sample_layers)]
     r = subprocess.run(cmd, env=env, capture_output=True, text=True)
@@ -312,7 +322,7 @@ def run_ours(args):
     world, rank, local = dist_setup(args)
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
-    cfg = workload_config(args.workload, args.n_max, args.layers)
+    cfg = workload_config(args.workload, args.n_max, args.layers, args.mode)
 
     # ---- inputs (seeded, synthetic; KV and Q drawn on the device)
     logits_h = W.make_logits(cfg)
@@ -335,7 +345,9 @@ def run_ours(args):
     r = taps.TapsRound(B=cfg.B, L=cfg.L, V=cfg.V, K=cfg.K, n_max=cfg.n_max, Hq=cfg.Hq,
                        Hkv=cfg.Hkv, D=cfg.D, max_ctx=int(ctx_h.max()), device=dev,
                        scorer_weights=torch.from_numpy(w["packed"]).to(dev), emb_dim=w["E"],
-                       hidden=w["H"], lambda1=cfg.lambda1, lambda2=cfg.lambda2, tau=cfg.tau)
+                       hidden=w["H"], lambda1=cfg.lambda1, lambda2=cfg.lambda2, tau=cfg.tau,
+                       mode=None if args.mode == "taps" else args.mode)
+    assert (r.lambda2, r.tau) == (cfg.lambda2, cfg.tau)
     # the stand-in target model's greedy tokens depend on the (deterministic) tree
     r.select(logits, root, ctx)
     torch.cuda.synchronize()
@@ -531,6 +543,7 @@ def run_ours(args):
                    "l2": f"inputs larger than L2: {cfg.layers} distinct KV layers, "
                          f"{kv_bytes / 1e9:.1f} GB per step",
                    "n_nodes": int(sel_h["n_nodes"][0]),
+                   "mode": args.mode,
                    "select_plus_one_layer_round_us": round(one_layer_us, 2),
                    "attention_stage_us_per_round": round(attn_ms * 1e3, 2)},
         "roofline": roofline,
@@ -559,7 +572,7 @@ def run_reference(args):
     world = int(os.environ.get("WORLD_SIZE", "1"))
     if rank != 0:
         return
-    cfg = workload_config(args.workload, args.n_max, args.layers)
+    cfg = workload_config(args.workload, args.n_max, args.layers, args.mode)
     cb = run_cpu_baseline(args, steps=args.steps, warmup=args.warmup, sample_layers=1)
     total = sum(cb["scaled_s"])
     value = args.steps / total
@@ -594,6 +607,9 @@ def main():
     ap.add_argument("--n-max", type=int, default=None, help="node budget (default: workload's)")
     ap.add_argument("--layers", type=int, default=None, help="layers (default: workload's)")
     ap.add_argument("--sample-layers", type=int, default=3)
+    ap.add_argument("--mode", default="taps",
+                    choices=["taps", "no_scorer", "budget_fill", "ddtree"],
+                    help="selection preset: TAPS, or one of its ablations")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-child", action="store_true", help=argparse.SUPPRESS)

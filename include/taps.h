@@ -61,7 +61,7 @@ typedef enum taps_status {
 } taps_status;
 
 enum { TAPS_F32 = 0, TAPS_BF16 = 1 };
-enum { TAPS_SCORER_MARGINAL = 0, TAPS_SCORER_MLP = 1 };
+enum { TAPS_SCORER_MARGINAL = 0, TAPS_SCORER_MLP = 1, TAPS_SCORER_MARGINAL_PRODUCT = 2 };
 enum { TAPS_DEVFAULT_PAGE = 1, TAPS_DEVFAULT_TIMEOUT = 2 };
 
 /* Limits (TAPS_ERR_UNSUPPORTED beyond them). */
@@ -147,6 +147,12 @@ int taps_topk_marginals_noalloc(const void* logits, int dtype, int64_t row_strid
  * Scorer (params->kind):
  *  TAPS_SCORER_MARGINAL  logit = topk_logp[b, d, j] (the paper's ablation that
  *                        ranks by the drafter's marginal confidence, Sec. 5.3).
+ *  TAPS_SCORER_MARGINAL_PRODUCT  no softmax: q_cond[b, d, i, j] =
+ *                        exp(topk_logp[b, d, j]) for every parent, so reach is
+ *                        the product of the path's marginal probabilities, the
+ *                        ranking of DDTree-style trees (Sec. 3.1, Limitation 1).
+ *                        With lambda2 = 0 and tau = 0 the selection then
+ *                        keeps the n_max paths of highest marginal probability.
  *  TAPS_SCORER_MLP       logit = w_lp * logp + w2 . relu(W1 f + b1) with
  *                        f = [E_tok[parent], E_tok[child], E_dep[d+1], logp,
  *                        entropy[b, d]] (Sec. 4.2 feature list). weights is a

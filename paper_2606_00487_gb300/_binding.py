@@ -26,7 +26,7 @@ lib = ctypes.CDLL(LIB_PATH)
 
 TAPS_OK = 0
 TAPS_F32, TAPS_BF16 = 0, 1
-TAPS_SCORER_MARGINAL, TAPS_SCORER_MLP = 0, 1
+TAPS_SCORER_MARGINAL, TAPS_SCORER_MLP, TAPS_SCORER_MARGINAL_PRODUCT = 0, 1, 2
 TAPS_DEVFAULT_PAGE = 1
 STATUS_NAMES = {0: "TAPS_OK", 1: "TAPS_ERR_INVALID_ARG", 2: "TAPS_ERR_UNSUPPORTED",
                 3: "TAPS_ERR_WORKSPACE", 4: "TAPS_ERR_CUDA", 5: "TAPS_ERR_DEVICE"}
@@ -160,6 +160,10 @@ def scorer_params(kind: str, weights: torch.Tensor | None = None, emb_dim=0, hid
                   max_depth=0) -> ScorerParams:
     if kind == "marginal":
         return ScorerParams(TAPS_SCORER_MARGINAL, 0, 0, 0, 0, None)
+    if kind == "marginal_product":
+        return ScorerParams(TAPS_SCORER_MARGINAL_PRODUCT, 0, 0, 0, 0, None)
+    if kind != "mlp":
+        raise ValueError(f"unknown scorer kind {kind!r}")
     _need(weights, torch.float32, name="scorer weights")
     F = 3 * emb_dim + 2
     expect = vocab * emb_dim + max_depth * emb_dim + hidden * F + 2 * hidden + 1

@@ -45,7 +45,7 @@ score_kernel(const int32_t* __restrict__ root_tok, const int32_t* __restrict__ i
   }
   __syncthreads();
 
-  if (kind == TAPS_SCORER_MARGINAL) {
+  if (kind != TAPS_SCORER_MLP) {
     for (int e = tid; e < np * K; e += kThreads) s_ell[e] = s_logp[e % K];
   } else {
     const float* tok_emb = w;
@@ -109,10 +109,13 @@ score_kernel(const int32_t* __restrict__ root_tok, const int32_t* __restrict__ i
   }
   __syncthreads();
 
-  // sibling-wise softmax, one thread per parent row
+  // sibling-wise softmax, one thread per parent row (the marginal-product
+  // kind takes each child's marginal probability as it is)
   float* out = q_cond + (static_cast<int64_t>(b) * L + d) * K * K;
   for (int i = tid; i < K; i += kThreads) {
-    if (i < np) {
+    if (i < np && kind == TAPS_SCORER_MARGINAL_PRODUCT) {
+      for (int j = 0; j < K; ++j) out[i * K + j] = expf(s_ell[i * K + j]);
+    } else if (i < np) {
       float m = -INFINITY;
       for (int j = 0; j < K; ++j) m = fmaxf(m, s_ell[i * K + j]);
       float sum = 0.f;
@@ -144,7 +147,7 @@ extern "C" int taps_score_reach(const int32_t* root_tok, const int32_t* topk_ids
         params->max_depth <= L)
       return TAPS_ERR_INVALID_ARG;
     if (E > TAPS_MAX_EMB || H > TAPS_MAX_HIDDEN) return TAPS_ERR_UNSUPPORTED;
-  } else if (kind != TAPS_SCORER_MARGINAL) {
+  } else if (kind != TAPS_SCORER_MARGINAL && kind != TAPS_SCORER_MARGINAL_PRODUCT) {
     return TAPS_ERR_INVALID_ARG;
   }
   size_t smem = sizeof(float) * (K * K + K + 2 * K * std::max(H, 1) + std::max(H, 1)) +

@@ -16,10 +16,29 @@ import torch
 from . import _binding as tb
 
 
+# Selection presets. "taps" is the method; "no_scorer" and "budget_fill" are
+# the two ablations of Sec. 5.3 (marginal confidence instead of the scorer;
+# the scorer without cost-aware pruning, lambda2 = 0 and tau = 0); "ddtree"
+# ranks paths by the product of the drafter's marginal probabilities and fills
+# the budget, the DDTree-style tree of Sec. 3.1.
+MODES = {
+    "taps": {"scorer_kind": "mlp"},
+    "no_scorer": {"scorer_kind": "marginal"},
+    "budget_fill": {"scorer_kind": "mlp", "lambda2": 0.0, "tau": 0.0},
+    "ddtree": {"scorer_kind": "marginal_product", "lambda2": 0.0, "tau": 0.0},
+}
+
+
 class TapsRound:
     def __init__(self, *, B, L, V, K, n_max, Hq, Hkv, D, max_ctx, device, scorer_kind="mlp",
                  scorer_weights=None, emb_dim=16, hidden=32, max_depth=None, lambda1=1.0,
-                 lambda2=0.1, tau=0.0):
+                 lambda2=0.1, tau=0.0, mode=None):
+        if mode is not None:
+            preset = MODES[mode]
+            scorer_kind = preset["scorer_kind"]
+            lambda2 = preset.get("lambda2", lambda2)
+            tau = preset.get("tau", tau)
+        self.mode = mode or "taps"
         dev = torch.device(device)
         self.B, self.L, self.V, self.K, self.n_max = B, L, V, K, n_max
         self.Hq, self.Hkv, self.D, self.max_ctx = Hq, Hkv, D, max_ctx
@@ -48,8 +67,8 @@ class TapsRound:
         self.ws_topk = torch.zeros(max(nb, 1), dtype=torch.uint8, device=dev)
         nb = tb.tree_verify_attn_workspace_bytes(B, n_max, Hq, Hkv, D, max_ctx)
         self.ws_attn = torch.zeros(max(nb, 1), dtype=torch.uint8, device=dev)
-        if scorer_kind == "marginal":
-            self.scorer = tb.scorer_params("marginal")
+        if scorer_kind in ("marginal", "marginal_product"):
+            self.scorer = tb.scorer_params(scorer_kind)
         else:
             self.scorer_weights = scorer_weights
             self.scorer = tb.scorer_params("mlp", scorer_weights, emb_dim, hidden, V,

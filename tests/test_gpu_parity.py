@@ -117,7 +117,10 @@ def _stage1_inputs(cfg, B=None):
 
 @pytest.mark.parametrize("name,kind", [("tiny", "mlp"), ("tiny", "marginal"),
                                        ("qwen3_8b", "mlp"), ("long", "mlp"),
-                                       ("qwen3_8b", "marginal"), ("llama31_8b", "mlp")])
+                                       ("qwen3_8b", "marginal"), ("llama31_8b", "mlp"),
+                                       ("tiny", "marginal_product"),
+                                       ("qwen3_8b", "marginal_product"),
+                                       ("long", "marginal_product")])
 def test_score_parity(taps, name, kind):
     cfg = W.CONFIGS[name]
     x, ids, logp, ent, root = _stage1_inputs(cfg, B=min(cfg.B, 2))
@@ -125,7 +128,7 @@ def test_score_parity(taps, name, kind):
     if kind == "mlp":
         sp = taps.scorer_params("mlp", dt(w["packed"]), w["E"], w["H"], w["V"], w["max_depth"])
     else:
-        sp = taps.scorer_params("marginal")
+        sp = taps.scorer_params(kind)
     q = taps.taps_score_reach(dt(root), dt(ids), dt(logp), dt(ent), sp)
     torch.cuda.synchronize()
     ref = O.score_qcond(root, ids, logp, ent, kind, w)
@@ -159,6 +162,29 @@ def test_select_parity(taps, name, n_max):
     q = O.score_qcond(root, ids, logp, ent, "mlp", w)
     ctx = W.make_ctx_lens(cfg, B=x.shape[0])
     _check_select(taps, q, ids, root, ctx, cfg.lambda1, cfg.lambda2, 0.0, n_max)
+
+
+@pytest.mark.parametrize("mode,name,n_max", [("budget_fill", "qwen3_8b", 64),
+                                             ("budget_fill", "long", 256),
+                                             ("no_scorer", "qwen3_8b", 64),
+                                             ("ddtree", "qwen3_8b", 64),
+                                             ("ddtree", "qwen3_8b", 512),
+                                             ("ddtree", "llama31_8b", 512)])
+def test_select_ablation_modes(taps, mode, name, n_max):
+    """Selection presets (Sec. 5.3 ablations, DDTree-style ranking of Sec. 3.1)
+    on the scorer output of that mode; budget-filling modes fill n_max."""
+    from paper_2606_00487_gb300.round import MODES
+    preset = MODES[mode]
+    cfg = W.CONFIGS[name]
+    x, ids, logp, ent, root = _stage1_inputs(cfg, B=min(cfg.B, 2))
+    w = W.make_scorer_weights(cfg)
+    q = O.score_qcond(root, ids, logp, ent, preset["scorer_kind"], w)
+    ctx = W.make_ctx_lens(cfg, B=x.shape[0])
+    l2 = preset.get("lambda2", cfg.lambda2)
+    tau = preset.get("tau", cfg.tau)
+    ref = _check_select(taps, q, ids, root, ctx, cfg.lambda1, l2, tau, n_max)
+    if l2 == 0.0 and tau == 0.0:
+        assert (ref["n_nodes"] == n_max).all()
 
 
 def test_select_batched_requests(taps):
@@ -475,10 +501,17 @@ def _near_tie_valid(tree, q_ref, ids, L, K, lambda1, lambda2, rtol=1e-5):
     return front_max <= sel_min * (1 + rtol)
 
 
-@pytest.mark.parametrize("name,n_max", [("tiny", 16), ("qwen3_8b", 64), ("qwen3_8b", 256),
-                                        ("llama31_8b", 64)])
-def test_round_end_to_end(taps, name, n_max):
-    cfg = W.CONFIGS[name]
+@pytest.mark.parametrize("name,n_max,mode", [("tiny", 16, "taps"), ("qwen3_8b", 64, "taps"),
+                                             ("qwen3_8b", 256, "taps"), ("llama31_8b", 64, "taps"),
+                                             ("qwen3_8b", 64, "ddtree"),
+                                             ("qwen3_8b", 64, "budget_fill"),
+                                             ("tiny", 16, "no_scorer")])
+def test_round_end_to_end(taps, name, n_max, mode):
+    from paper_2606_00487_gb300.round import MODES
+    preset = MODES[mode]
+    kind = preset["scorer_kind"]
+    cfg = W.CONFIGS[name].with_(lambda2=preset.get("lambda2", W.CONFIGS[name].lambda2),
+                                tau=preset.get("tau", W.CONFIGS[name].tau))
     x = W.make_logits(cfg)
     root, ctx = W.make_root_tokens(cfg), W.make_ctx_lens(cfg)
     w = W.make_scorer_weights(cfg)
@@ -486,13 +519,14 @@ def test_round_end_to_end(taps, name, n_max):
     r = taps.TapsRound(B=cfg.B, L=cfg.L, V=cfg.V, K=cfg.K, n_max=n_max, Hq=cfg.Hq, Hkv=cfg.Hkv,
                        D=cfg.D, max_ctx=int(ctx.max()), device=DEV,
                        scorer_weights=dt(w["packed"]), emb_dim=w["E"], hidden=w["H"],
-                       lambda1=cfg.lambda1, lambda2=cfg.lambda2, tau=cfg.tau)
+                       lambda1=cfg.lambda1, mode=mode)
+    assert (r.lambda2, r.tau) == (cfg.lambda2, cfg.tau)
     xd = dt(x).to(torch.float32 if cfg.logits_dtype == "f32" else torch.bfloat16)
     r.select(xd, dt(root), dt(ctx))
     torch.cuda.synchronize()
     ids, logp, lse, ent = O.topk_marginals(x, cfg.K)
     np.testing.assert_array_equal(host(r.ids), ids)
-    q_ref = O.score_qcond(root, ids, logp, ent, "mlp", w)
+    q_ref = O.score_qcond(root, ids, logp, ent, kind, w)
     np.testing.assert_allclose(host(r.q_cond), q_ref, rtol=1e-4, atol=1e-6)
     # topology: bit-exact given the GPU's own q_cond, near-tie valid under the oracle's
     gq = host(r.q_cond)
@@ -522,6 +556,14 @@ def test_round_end_to_end(taps, name, n_max):
     r.accept(dt(tt))
     torch.cuda.synchronize()
     a = O.accept(sel["parent"], sel["token"], sel["n_nodes"], tt, cfg.L)
+    np.testing.assert_array_equal(host(r.accept_len), a[0])
+    np.testing.assert_array_equal(host(r.accepted_nodes), a[1])
+    np.testing.assert_array_equal(host(r.bonus_tok), a[2])
+    # the same acceptance from verify logits whose greedy tokens are the targets
+    r.accept_len.fill_(-7)
+    r.accept_greedy(W.make_verify_logits_torch(cfg, dt(tt), DEV))
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(host(r.target_tok), tt)
     np.testing.assert_array_equal(host(r.accept_len), a[0])
     np.testing.assert_array_equal(host(r.accepted_nodes), a[1])
     np.testing.assert_array_equal(host(r.bonus_tok), a[2])
