@@ -691,16 +691,24 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
   float2* stat = reinterpret_cast<float2*>(smem + S::kStat);
   if (got && threadIdx.x < re - rb) {
     // per row: the cluster-wide max M, each chunk's weight l_q 2^(m_q - M)
-    // (in place of m_q) and the total L
+    // (in place of m_q) and the total L. Unrolled to the largest cluster, so
+    // that every peer's (max, sum) is loaded at once.
     const int i = threadIdx.x;
+    float2 ml[kMaxCluster];
+#pragma unroll
+    for (int q = 0; q < kMaxCluster; ++q)
+      ml[q] = q < cs ? rml[q * per + i] : make_float2(-INFINITY, 0.f);
     float M = -INFINITY;
-    for (int q = 0; q < cs; ++q) M = fmaxf(M, rml[q * per + i].x);
+#pragma unroll
+    for (int q = 0; q < kMaxCluster; ++q) M = fmaxf(M, ml[q].x);
     float L = 0.f;
-    for (int q = 0; q < cs; ++q) {
-      const float2 ml = rml[q * per + i];
-      const float w = ml.y > 0.f ? ml.y * ex2_approx(ml.x - M) : 0.f;
-      rml[q * per + i].x = w;
-      L += w;
+#pragma unroll
+    for (int q = 0; q < kMaxCluster; ++q) {
+      if (q < cs) {
+        const float w = ml[q].y > 0.f ? ml[q].y * ex2_approx(ml[q].x - M) : 0.f;
+        rml[q * per + i].x = w;
+        L += w;
+      }
     }
     stat[i] = make_float2(M, L);
   }
