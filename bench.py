@@ -331,14 +331,21 @@ def run_ours(args):
     bt_h, num_pages = W.make_block_table(cfg, ctx_h)
     y = W.make_target_sequence(cfg, logits_h)
     ldt = torch.bfloat16 if cfg.logits_dtype == "bf16" else torch.float32
-    logits = torch.from_numpy(logits_h).to(dev).to(ldt)
-    root, ctx = torch.from_numpy(root_h).to(dev), torch.from_numpy(ctx_h).to(dev)
+    # the round's per-step inputs live in one staging buffer (one upload per round)
+    inp = taps.RoundInputs(B=cfg.B, L=cfg.L, V=cfg.V, n_max=cfg.n_max, Hq=cfg.Hq, D=cfg.D,
+                           layers=cfg.layers, logits_dtype=ldt, device=dev)
+    logits = inp.dev["logits"]
+    logits.copy_(torch.from_numpy(logits_h).to(dev).to(ldt))
+    root = inp.dev["root_tok"]
+    root.copy_(torch.from_numpy(root_h).to(dev))
+    ctx = torch.from_numpy(ctx_h).to(dev)
     bt = torch.from_numpy(bt_h).to(dev)
     layers = []
     for layer in range(cfg.layers):
         kc, vc = W.make_kv_torch(cfg, num_pages, layer, dev)
         kc, vc = taps.taps_pack_kv_pages(kc), taps.taps_pack_kv_pages(vc)   # TAPS page layout
-        q = W.make_q_torch(cfg, cfg.B, cfg.n_max, layer, dev)
+        q = inp.dev["q"][layer]
+        q.copy_(W.make_q_torch(cfg, cfg.B, cfg.n_max, layer, dev))
         layers.append((q, kc, vc, bt))
     outs = [torch.empty_like(layers[0][0]) for _ in range(cfg.layers)]
 
@@ -353,7 +360,8 @@ def run_ours(args):
     torch.cuda.synchronize()
     sel_h = {k: v.cpu().numpy() for k, v in r.sel.items()}
     tt_h = W.target_tokens_for_tree(y, sel_h["depth"], sel_h["n_nodes"])
-    target = torch.from_numpy(tt_h).to(dev)
+    target = inp.dev["target_tok"]
+    target.copy_(torch.from_numpy(tt_h).to(dev))
 
     # ---- capture the round as three graphs
     s = torch.cuda.Stream(device=dev)
@@ -363,10 +371,11 @@ def run_ours(args):
             r.run(logits, root, ctx, layers, outs, target)
     torch.cuda.current_stream(dev).wait_stream(s)
     torch.cuda.synchronize()
-    g_pre, g_attn, g_post = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
+    g_pre, g_post = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
     with torch.cuda.graph(g_pre, stream=s):
         r.select(logits, root, ctx)
-    with torch.cuda.graph(g_attn, stream=s):
+    g_attn_all = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g_attn_all, stream=s):
         for (q, kc, vc, b_t), o in zip(layers, outs):
             r.verify_layer(q, kc, vc, b_t, ctx, o)
     with torch.cuda.graph(g_post, stream=s):
@@ -379,7 +388,7 @@ def run_ours(args):
         g_pre.replay()
         if ev_a is not None:
             ev_a.record(stream)
-        g_attn.replay()
+        g_attn_all.replay()
         if ev_b is not None:
             ev_b.record(stream)
         g_post.replay()
@@ -467,26 +476,30 @@ def run_ours(args):
     # ---- end to end through the public API with host buffers
     e2e = None
     if not args.no_e2e:
-        pin = lambda t: t.cpu().pin_memory()
-        logits_pin = pin(logits)
-        q_pin = [pin(q) for (q, _, _, _) in layers]
-        target_pin = pin(target)
-        res_pin = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
-                   for t in (r.sel["n_nodes"], r.accept_len, r.accepted_nodes, r.bonus_tok)]
-        h2d = (logits_pin.numel() * logits_pin.element_size()
-               + sum(t.numel() * t.element_size() for t in q_pin)
-               + target_pin.numel() * target_pin.element_size())
-        d2h = sum(t.numel() * t.element_size() for t in res_pin)
+        # the host staging buffer holds every input of a round (logits, root
+        # tokens, the 36 layers' tree queries, target tokens): one upload per
+        # round, then the round, then one read of its results
+        # The head (logits, root and target tokens) goes first on the compute
+        # stream; the queries of all layers travel on a copy stream while the
+        # selection stages run, and verification waits for them.
+        torch.cuda.synchronize()
+        inp.host_buf.copy_(inp.device_buf)
+        res_pin = torch.empty(r.results.shape, dtype=r.results.dtype, pin_memory=True)
+        h2d = inp.nbytes
+        d2h = res_pin.numel() * res_pin.element_size()
+        copy_stream = torch.cuda.Stream(device=dev)
+        q_ready = torch.cuda.Event()
 
         def e2e_step():
-            logits.copy_(logits_pin, non_blocking=True)
-            for (q, _, _, _), qp in zip(layers, q_pin):
-                q.copy_(qp, non_blocking=True)
-            target.copy_(target_pin, non_blocking=True)
-            step()
-            for dst, src in zip(res_pin, (r.sel["n_nodes"], r.accept_len, r.accepted_nodes,
-                                          r.bonus_tok)):
-                dst.copy_(src, non_blocking=True)
+            copy_stream.wait_stream(stream)        # the previous round is done with the queries
+            inp.upload_head(stream)
+            inp.upload_queries(copy_stream)
+            q_ready.record(copy_stream)
+            g_pre.replay()
+            stream.wait_event(q_ready)
+            g_attn_all.replay()
+            g_post.replay()
+            r.download(res_pin, stream)
             stream.synchronize()
 
         for _ in range(args.warmup):

@@ -14,9 +14,9 @@ from ._binding import (LIB_PATH, TAPS_DEVFAULT_PAGE, TapsError, lib, scorer_para
                        topk_marginals_workspace_bytes, tree_verify_attn_workspace_bytes,
                        taps_target_greedy_accept, target_greedy_accept_workspace_bytes,
                        taps_compact_accepted_kv)
-from .round import MODES, TapsRound  # noqa: F401
+from .round import MODES, RoundInputs, TapsRound  # noqa: F401
 
 __all__ = ["taps_topk_marginals", "taps_score_reach", "taps_select_subtree",
-           "taps_build_tree_mask", "taps_tree_verify_attn", "taps_accept", "TapsRound",
+           "taps_build_tree_mask", "taps_tree_verify_attn", "taps_accept", "TapsRound", "RoundInputs",
            "TapsError", "scorer_params", "MODES", "taps_target_greedy_accept",
            "taps_compact_accepted_kv"]

@@ -50,15 +50,18 @@ class TapsRound:
         self.lse = torch.empty((B, L), dtype=f32, device=dev)
         self.entropy = torch.empty((B, L), dtype=f32, device=dev)
         self.q_cond = torch.empty((B, L, K, K), dtype=f32, device=dev)
-        self.sel = {"n_nodes": torch.empty(B, dtype=i32, device=dev)}
+        # the round's results (n_nodes, accept_len, bonus_tok, accepted_nodes)
+        # live in one int32 buffer, so that the host reads them in one copy
+        self.results = torch.empty(3 * B + B * (L + 1), dtype=i32, device=dev)
+        self.sel = {"n_nodes": self.results[0:B]}
         for k in ("parent", "depth", "token", "slot", "pos_id"):
             self.sel[k] = torch.empty((B, n_max), dtype=i32, device=dev)
         for k in ("reach", "utility"):
             self.sel[k] = torch.empty((B, n_max), dtype=f32, device=dev)
         self.mask = torch.empty((B, n_max, (n_max + 31) // 32), dtype=i32, device=dev)
-        self.accept_len = torch.empty(B, dtype=i32, device=dev)
-        self.accepted_nodes = torch.empty((B, L + 1), dtype=i32, device=dev)
-        self.bonus_tok = torch.empty(B, dtype=i32, device=dev)
+        self.accept_len = self.results[B:2 * B]
+        self.accepted_nodes = self.results[3 * B:].view(B, L + 1)
+        self.bonus_tok = self.results[2 * B:3 * B]
         self.status = torch.zeros(1, dtype=i32, device=dev)
         self.target_tok = torch.empty((B, n_max), dtype=i32, device=dev)
         nb = tb.target_greedy_accept_workspace_bytes(B, n_max)
@@ -114,9 +117,74 @@ class TapsRound:
                                     self.accepted_nodes, self.accept_len, status=self.status,
                                     stream=stream)
 
+    def download(self, host_results, stream=None):
+        """Copy the round's results (n_nodes, accept_len, bonus_tok, then
+        accepted_nodes row by row, int32) into a pinned host tensor of
+        results.numel() elements: one device-to-host copy."""
+        with torch.cuda.stream(stream or torch.cuda.current_stream(self.device)):
+            host_results.copy_(self.results, non_blocking=True)
+
     def run(self, logits, root_tok, ctx_len, layers, outs, target_tok, stream=None):
         """layers: list of (q, k_cache, v_cache, block_table); outs: one output per layer."""
         self.select(logits, root_tok, ctx_len, stream)
         for (q, kc, vc, bt), o in zip(layers, outs):
             self.verify_layer(q, kc, vc, bt, ctx_len, o, stream)
         self.accept(target_tok, stream)
+
+
+class RoundInputs:
+    """A round's inputs in one device buffer mirrored by one pinned host
+    buffer: the drafter's logits [B, L, V], the root tokens [B], the target's
+    greedy tokens [B, n_max] (the head, needed from the first stage on), then
+    every layer's tree-node queries [layers, B, n_max, Hq, D] bf16 (needed
+    only by verification). ``dev[name]`` and ``host[name]`` are views of the
+    two buffers. upload() copies everything at once; upload_head() and
+    upload_queries() copy the two parts, so that the queries can travel on
+    another stream while the selection stages run."""
+
+    def __init__(self, *, B, L, V, n_max, Hq, D, layers, logits_dtype, device):
+        parts = [("logits", (B, L, V), logits_dtype),
+                 ("root_tok", (B,), torch.int32),
+                 ("target_tok", (B, n_max), torch.int32),
+                 ("q", (layers, B, n_max, Hq, D), torch.bfloat16)]
+        offs, o = {}, 0
+        for name, shape, dt in parts:
+            n = 1
+            for x in shape:
+                n *= x
+            nbytes = n * torch.empty((), dtype=dt).element_size()
+            offs[name] = (o, nbytes, shape, dt)
+            o += (nbytes + 255) // 256 * 256
+        self.nbytes = o
+        self.payload_bytes = sum(v[1] for v in offs.values())
+        self.device_buf = torch.empty(o, dtype=torch.uint8, device=device)
+        self.host_buf = torch.empty(o, dtype=torch.uint8, pin_memory=True)
+
+        def views(buf):
+            return {name: buf[a:a + nb].view(dt).view(shape)
+                    for name, (a, nb, shape, dt) in offs.items()}
+
+        self.dev = views(self.device_buf)
+        self.host = views(self.host_buf)
+        self.head_bytes = offs["q"][0]
+        self.layers = layers
+        self.layer_bytes = offs["q"][1] // layers
+
+    def _copy(self, a, b, stream):
+        with torch.cuda.stream(stream or torch.cuda.current_stream(self.device_buf.device)):
+            self.device_buf[a:b].copy_(self.host_buf[a:b], non_blocking=True)
+
+    def upload(self, stream=None):
+        """Host buffer -> device buffer, asynchronously on ``stream``."""
+        self._copy(0, self.nbytes, stream)
+
+    def upload_head(self, stream=None):
+        """Logits, root tokens and target tokens only."""
+        self._copy(0, self.head_bytes, stream)
+
+    def upload_queries(self, stream=None, first=0, last=None):
+        """The tree-node queries of layers [first, last) only (default: all)."""
+        last = self.layers if last is None else last
+        a = self.head_bytes + first * self.layer_bytes
+        b = self.nbytes if last == self.layers else self.head_bytes + last * self.layer_bytes
+        self._copy(a, b, stream)

@@ -234,3 +234,42 @@ def test_compact_bad_page_sets_status(taps):
     taps.taps_compact_accepted_kv(kd, vd, dt(bt), dt(ctx), dt(path), dt(alen), status=status)
     torch.cuda.synchronize()
     assert int(status.item()) & taps.TAPS_DEVFAULT_PAGE
+
+
+def test_round_inputs_single_upload_and_results_download(taps):
+    """Inputs staged in one pinned buffer reach the device views in one copy;
+    a round run on those views matches the oracle, and its results come back
+    in one copy in the documented order."""
+    cfg = W.CONFIGS["tiny"]
+    B, n_max = 1, 16
+    x = W.make_logits(cfg)
+    root, ctx = W.make_root_tokens(cfg), W.make_ctx_lens(cfg)
+    inp = taps.RoundInputs(B=B, L=cfg.L, V=cfg.V, n_max=n_max, Hq=cfg.Hq, D=cfg.D, layers=2,
+                           logits_dtype=torch.float32, device=DEV)
+    inp.host["logits"].copy_(torch.from_numpy(x))
+    inp.host["root_tok"].copy_(torch.from_numpy(root))
+    inp.host["target_tok"].fill_(-1)
+    inp.upload()
+    torch.cuda.synchronize()
+    assert torch.equal(inp.dev["logits"].cpu(), torch.from_numpy(x))
+    r = taps.TapsRound(B=B, L=cfg.L, V=cfg.V, K=cfg.K, n_max=n_max, Hq=cfg.Hq, Hkv=cfg.Hkv,
+                       D=cfg.D, max_ctx=int(ctx.max()), device=DEV, mode="no_scorer")
+    r.select(inp.dev["logits"], inp.dev["root_tok"], dt(ctx))
+    torch.cuda.synchronize()
+    ids, logp, _, ent = O.topk_marginals(x, cfg.K)
+    q = O.score_qcond(root, ids, logp, ent, "marginal")
+    sel = O.select_subtree(host(r.q_cond), ids, root, ctx, cfg.lambda1, cfg.lambda2, cfg.tau,
+                           n_max)
+    y = W.make_target_sequence(cfg, x)
+    tt = W.target_tokens_for_tree(y, sel["depth"], sel["n_nodes"])
+    inp.host["target_tok"].copy_(torch.from_numpy(tt))
+    inp.upload()
+    r.accept(inp.dev["target_tok"])
+    res = torch.empty(r.results.shape, dtype=torch.int32, pin_memory=True)
+    r.download(res)
+    torch.cuda.synchronize()
+    a_len, nodes, bonus = O.accept(sel["parent"], sel["token"], sel["n_nodes"], tt, cfg.L)
+    res = res.numpy()
+    np.testing.assert_allclose(host(r.q_cond), q, rtol=1e-5, atol=1e-7)
+    assert res[0] == sel["n_nodes"][0] and res[1] == a_len[0] and res[2] == bonus[0]
+    np.testing.assert_array_equal(res[3:].reshape(B, cfg.L + 1), nodes)
