@@ -17,6 +17,7 @@ accept_kernel(const int32_t* __restrict__ parent, const int32_t* __restrict__ to
               const int32_t* __restrict__ n_nodes, const int32_t* __restrict__ target_tok,
               int n_max, int L, int32_t* __restrict__ accept_len,
               int32_t* __restrict__ accepted_nodes, int32_t* __restrict__ bonus_tok) {
+  dep_enter();
   __shared__ int32_t s_par[TAPS_MAX_NODES], s_tok[TAPS_MAX_NODES], s_tt[TAPS_MAX_NODES];
   __shared__ int32_t s_match[TAPS_MAX_NODES];
   const int b = blockIdx.x;
@@ -46,7 +47,9 @@ extern "C" int taps_accept(const int32_t* parent, const int32_t* token, const in
     return TAPS_ERR_INVALID_ARG;
   if (B <= 0 || n_max <= 0 || L < 0) return TAPS_ERR_INVALID_ARG;
   if (n_max > TAPS_MAX_NODES || L > TAPS_MAX_L || B > 65535) return TAPS_ERR_UNSUPPORTED;
-  accept_kernel<<<B, kThreads, 0, static_cast<cudaStream_t>(stream)>>>(
-      parent, token, n_nodes, target_tok, n_max, L, accept_len, accepted_nodes, bonus_tok);
+  if (launch_dep(accept_kernel, dim3(B), dim3(kThreads), 0, static_cast<cudaStream_t>(stream),
+                 parent, token, n_nodes, target_tok, n_max, L, accept_len, accepted_nodes,
+                 bonus_tok) != cudaSuccess)
+    return TAPS_ERR_CUDA;
   return launch_status();
 }

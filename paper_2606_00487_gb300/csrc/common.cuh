@@ -5,6 +5,8 @@
 #include <cuda_bf16.h>
 #include <stdint.h>
 
+#include <utility>
+
 #include "taps.h"
 
 namespace taps {
@@ -15,6 +17,33 @@ constexpr int kTargetSms = 152;
 constexpr unsigned kFullMask = 0xffffffffu;
 
 inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// Programmatic dependent launch. Every kernel of the library is launched
+// with programmatic stream serialisation, so that its launch and prologue may
+// overlap the tail of the kernel before it on the stream. dep_enter() is the
+// first statement of every such kernel: it waits until the previous grid has
+// completed and its memory is visible (so no input is read and no output
+// written before that), then lets the next kernel on the stream be launched.
+__device__ __forceinline__ void dep_enter() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_dep(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                              cudaStream_t stream, Args&&... args) {
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
 
 inline int launch_status() {
   cudaError_t e = cudaGetLastError();

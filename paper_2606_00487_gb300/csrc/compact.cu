@@ -36,6 +36,7 @@ compact_kernel(LayerBases bases, int B, int Hkv, int D, int64_t num_pages,
                const int32_t* __restrict__ block_table, int max_pages,
                const int32_t* __restrict__ ctx_len, const int32_t* __restrict__ accepted_nodes,
                const int32_t* __restrict__ accept_len, int L, int32_t* status) {
+  dep_enter();
   const int lkv = blockIdx.x / B;            // 2 * layer + (0 K, 1 V)
   const int b = blockIdx.x - lkv * B;
   const int h = blockIdx.y;
@@ -111,8 +112,9 @@ extern "C" int taps_compact_accepted_kv(void* const* k_layers, void* const* v_la
     bases.p[2 * l + 1] = static_cast<uint4*>(v_layers[l]);
   }
   const dim3 grid(static_cast<unsigned>(B * 2 * num_layers), static_cast<unsigned>(Hkv));
-  compact_kernel<<<grid, kThreads, 0, static_cast<cudaStream_t>(stream)>>>(
-      bases, B, Hkv, D, num_pages, block_table, max_pages, ctx_len, accepted_nodes, accept_len,
-      L, status);
+  if (launch_dep(compact_kernel, grid, dim3(kThreads), 0, static_cast<cudaStream_t>(stream),
+                 bases, B, Hkv, D, num_pages, block_table, max_pages, ctx_len, accepted_nodes,
+                 accept_len, L, status) != cudaSuccess)
+    return TAPS_ERR_CUDA;
   return launch_status();
 }

@@ -15,6 +15,7 @@ constexpr int kThreads = 256;
 __global__ void __launch_bounds__(kThreads)
 mask_kernel(const int32_t* __restrict__ parent, const int32_t* __restrict__ n_nodes, int n_max,
             int W, uint32_t* __restrict__ mask) {
+  dep_enter();
   const int b = blockIdx.x;
   const int n = min(max(n_nodes[b], 0), n_max);
   const int32_t* pb = parent + static_cast<int64_t>(b) * n_max;
@@ -48,7 +49,8 @@ extern "C" int taps_build_tree_mask(const int32_t* parent, const int32_t* n_node
   if (B <= 0 || n_max <= 0) return TAPS_ERR_INVALID_ARG;
   if (n_max > TAPS_MAX_NODES || B > 65535) return TAPS_ERR_UNSUPPORTED;
   const int W = (n_max + 31) / 32;
-  mask_kernel<<<B, kThreads, 0, static_cast<cudaStream_t>(stream)>>>(parent, n_nodes, n_max, W,
-                                                                       mask);
+  if (launch_dep(mask_kernel, dim3(B), dim3(kThreads), 0, static_cast<cudaStream_t>(stream),
+                 parent, n_nodes, n_max, W, mask) != cudaSuccess)
+    return TAPS_ERR_CUDA;
   return launch_status();
 }

@@ -20,6 +20,7 @@ score_kernel(const int32_t* __restrict__ root_tok, const int32_t* __restrict__ i
              const float* __restrict__ logp, const float* __restrict__ entropy, int L, int K,
              int kind, int E, int H, int vocab, int max_depth, const float* __restrict__ w,
              float* __restrict__ q_cond) {
+  dep_enter();
   extern __shared__ float sm[];
   const int d = blockIdx.x;
   const int b = blockIdx.y;
@@ -153,8 +154,10 @@ extern "C" int taps_score_reach(const int32_t* root_tok, const int32_t* topk_ids
   size_t smem = sizeof(float) * (K * K + K + 2 * K * std::max(H, 1) + std::max(H, 1)) +
                 sizeof(int) * 2 * K;
   dim3 grid(L, B);
-  score_kernel<<<grid, kThreads, smem, static_cast<cudaStream_t>(stream)>>>(
-      root_tok, topk_ids, topk_logp, entropy, L, K, kind, E, H, params->vocab,
-      params->max_depth, params->weights, q_cond);
+  if (launch_dep(score_kernel, grid, dim3(kThreads), smem, static_cast<cudaStream_t>(stream),
+                 root_tok, topk_ids, topk_logp, entropy, L, K, kind, E, H, params->vocab,
+                 params->max_depth, static_cast<const float*>(params->weights), q_cond) !=
+      cudaSuccess)
+    return TAPS_ERR_CUDA;
   return launch_status();
 }

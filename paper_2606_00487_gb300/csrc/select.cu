@@ -113,6 +113,7 @@ select_kernel(const float* __restrict__ q_cond, const int* __restrict__ ids,
               int32_t* __restrict__ depth_out, int32_t* __restrict__ token_out,
               int32_t* __restrict__ slot_out, int32_t* __restrict__ pos_out,
               float* __restrict__ reach_out, float* __restrict__ util_out) {
+  dep_enter();
   extern __shared__ __align__(16) char smem_raw[];
   const int b = blockIdx.x;
   const int lane = threadIdx.x;
@@ -279,9 +280,10 @@ int launch_select(const float* q_cond, const int32_t* topk_ids, const int32_t* r
       cudaFuncSetAttribute(select_kernel<SPL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            static_cast<int>(smem)) != cudaSuccess)
     return TAPS_ERR_CUDA;
-  select_kernel<SPL><<<B, 32, smem, stream>>>(q_cond, topk_ids, root_tok, ctx_len, L, K, l1, l2,
-                                               tau, n_max, n_nodes, parent, depth, token, slot,
-                                               pos_id, reach, utility);
+  if (launch_dep(select_kernel<SPL>, dim3(B), dim3(32), smem, stream, q_cond, topk_ids, root_tok,
+                 ctx_len, L, K, l1, l2, tau, n_max, n_nodes, parent, depth, token, slot, pos_id,
+                 reach, utility) != cudaSuccess)
+    return TAPS_ERR_CUDA;
   return launch_status();
 }
 

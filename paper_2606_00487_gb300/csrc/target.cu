@@ -73,6 +73,7 @@ target_greedy_accept_kernel(const T* __restrict__ logits, int64_t row_stride, in
                             int32_t* __restrict__ accepted_nodes,
                             int32_t* __restrict__ bonus_tok, unsigned long long* keys,
                             unsigned* tickets) {
+  dep_enter();
   constexpr int W = kVec ? static_cast<int>(16 / sizeof(T)) : 1;
   const int row = blockIdx.x / plan.splits;
   const int split = blockIdx.x - row * plan.splits;
@@ -226,11 +227,11 @@ void launch(const void* logits, int64_t row_stride, int B, int n_max, int V,
   const TargetPlan p = make_target_plan(B, n_max, V, W);
   const TargetWs w = target_ws(B, n_max);
   const int64_t grid = static_cast<int64_t>(B) * n_max * p.splits;
-  target_greedy_accept_kernel<T, kVec><<<static_cast<unsigned>(grid), kThreads, 0, s>>>(
-      static_cast<const T*>(logits), row_stride, n_max, V, p, parent, token, n_nodes, L,
-      target_tok, accept_len, accepted_nodes, bonus_tok,
-      reinterpret_cast<unsigned long long*>(ws + w.keys),
-      reinterpret_cast<unsigned*>(ws + w.tickets));
+  launch_dep(target_greedy_accept_kernel<T, kVec>, dim3(static_cast<unsigned>(grid)),
+             dim3(kThreads), 0, s, static_cast<const T*>(logits), row_stride, n_max, V, p, parent,
+             token, n_nodes, L, target_tok, accept_len, accepted_nodes, bonus_tok,
+             reinterpret_cast<unsigned long long*>(ws + w.keys),
+             reinterpret_cast<unsigned*>(ws + w.tickets));
 }
 
 }  // namespace

@@ -193,6 +193,7 @@ topk_marginals_kernel(const T* __restrict__ logits, int64_t row_stride, int V, i
                       int vec_ok, int32_t* __restrict__ ids, float* __restrict__ logp,
                       float* __restrict__ lse, float* __restrict__ ent, float4* ws_stats,
                       uint64_t* ws_keys, unsigned* tickets) {
+  dep_enter();
   constexpr int VE = 16 / sizeof(T);
   __shared__ uint64_t s_cand[kMaxChunks * 32];
   __shared__ uint64_t s_top[32];
@@ -406,9 +407,9 @@ void launch(const void* logits, int64_t row_stride, const Plan& p, int V, int K,
   float4* st = p.chunks > 1 ? reinterpret_cast<float4*>(ws + w.stats) : nullptr;
   uint64_t* keys = p.chunks > 1 ? reinterpret_cast<uint64_t*>(ws + w.keys) : nullptr;
   unsigned* tk = p.chunks > 1 ? reinterpret_cast<unsigned*>(ws + w.tickets) : nullptr;
-  topk_marginals_kernel<KP, T><<<grid, kThreads, 0, s>>>(
-      static_cast<const T*>(logits), row_stride, V, K, p.chunks, vec_ok, ids, logp, lse, ent,
-      st, keys, tk);
+  launch_dep(topk_marginals_kernel<KP, T>, grid, dim3(kThreads), 0, s,
+             static_cast<const T*>(logits), row_stride, V, K, p.chunks, vec_ok, ids, logp, lse,
+             ent, st, keys, tk);
 }
 
 template <typename T>
