@@ -23,6 +23,9 @@ namespace {
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
 constexpr int kMaxChunks = 64;
+constexpr int kRing = 4;                       // tiles per thread in its copy ring
+constexpr int kFewKeys = 8;                    // at most this many tile keys: insert one by one
+constexpr size_t kRingBytes = static_cast<size_t>(kRing) * 2 * kThreads * 16;
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 
@@ -40,8 +43,8 @@ Plan make_plan(int B, int L, int V, int K) {
   Plan p;
   p.rows = B * L;
   p.kp = round_kp(K);
-  // two CTAs per SM: the 256-thread CTAs hold about 80 registers per thread,
-  // so three fit an SM, and one wave of two per SM avoids a second wave
+  // two CTAs per SM (registers and the 64 KB copy ring each allow two), in
+  // one wave where the rows are few
   int want = (2 * kTargetSms + p.rows - 1) / p.rows;
   int maxc = std::max(1, V / 2048);
   p.chunks = std::max(1, std::min(want, std::min(maxc, kMaxChunks)));
@@ -194,12 +197,19 @@ topk_marginals_kernel(const T* __restrict__ logits, int64_t row_stride, int V, i
                       float* __restrict__ lse, float* __restrict__ ent, float4* ws_stats,
                       uint64_t* ws_keys, unsigned* tickets) {
   dep_enter();
+  extern __shared__ __align__(16) unsigned char dyn_smem[];   // copy ring (vector path)
   constexpr int VE = 16 / sizeof(T);
   __shared__ uint64_t s_cand[kMaxChunks * 32];
   __shared__ uint64_t s_top[32];
   __shared__ uint64_t s_part[kWarps * 32];
   __shared__ Stats s_wstats[kWarps];
   __shared__ int s_last;
+  // The largest K-th key any warp of this CTA holds: at least KP keys of the
+  // row are >= it, so a key below it can be in no top-K (keys are unique, and
+  // the key itself sits in the list of the warp that holds it)
+  __shared__ unsigned long long s_thr;
+  if (threadIdx.x == 0) s_thr = 0ull;
+  __syncthreads();
 
   const int row = blockIdx.y;
   const int chunk = blockIdx.x;
@@ -224,7 +234,58 @@ topk_marginals_kernel(const T* __restrict__ logits, int64_t row_stride, int V, i
     uint64_t lm = 0;
 #pragma unroll
     for (int i = 0; i < EPT; ++i) lm = k[i] > lm ? k[i] : lm;
-    if (!__any_sync(kFullMask, lm > kth)) return;
+    const uint64_t shared_thr = *reinterpret_cast<volatile unsigned long long*>(&s_thr);
+    const uint64_t thr = shared_thr > kth ? shared_thr : kth;
+    if (!__any_sync(kFullMask, lm > thr)) return;
+    // Insert the candidates c4[0 .. cnt) of every lane into the lane-sorted
+    // running list, one key after another. Lane r < KP holds the r-th
+    // largest; a new key goes to position pos = (entries above it), and the
+    // entries from pos on shift one lane down (the K-th falls off).
+    auto insert_all = [&](const uint64_t (&c4)[4], int cnt) {
+      unsigned todo = __ballot_sync(kFullMask, cnt > 0);
+      while (todo) {
+        const int src = __ffs(todo) - 1;
+        todo &= todo - 1;
+        const int n_src = __shfl_sync(kFullMask, cnt, src);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          if (j < n_src) {
+            const uint64_t key = __shfl_sync(kFullMask, c4[j], src);
+            const unsigned above = __ballot_sync(kFullMask, lane < KP && run > key);
+            const int pos = __popc(above);
+            const uint64_t up = __shfl_up_sync(kFullMask, run, 1);
+            // (an earlier insertion may have raised the K-th above this key)
+            if (pos < KP) {
+              if (lane < KP && lane > pos) run = up;
+              if (lane == pos) run = key;
+            }
+          }
+        }
+      }
+      kth = __shfl_sync(kFullMask, run, KP - 1);
+      if (lane == 0 && kth > thr) atomicMax(&s_thr, static_cast<unsigned long long>(kth));
+    };
+    {
+      // Few candidates (the usual case once the list has filled): insert the
+      // keys above the threshold directly.
+      uint64_t c4[4] = {0ull, 0ull, 0ull, 0ull};
+      int cnt = 0;
+#pragma unroll
+      for (int i = 0; i < EPT; ++i) {
+        if (k[i] > thr) {
+          c4[3] = c4[2];
+          c4[2] = c4[1];
+          c4[1] = c4[0];
+          c4[0] = k[i];
+          ++cnt;
+        }
+      }
+      const int total = __reduce_add_sync(kFullMask, static_cast<unsigned>(cnt));
+      if (total <= kFewKeys && !__any_sync(kFullMask, cnt > 4)) {
+        insert_all(c4, cnt);
+        return;
+      }
+    }
     int rank = 0;   // lane maxima above this lane's (keys are unique, 0 = none)
 #pragma unroll
     for (int l = 0; l < 32; ++l) rank += __shfl_sync(kFullMask, lm, l) > lm ? 1 : 0;
@@ -234,7 +295,7 @@ topk_marginals_kernel(const T* __restrict__ logits, int64_t row_stride, int V, i
     int cnt = 0;
 #pragma unroll
     for (int i = 0; i < EPT; ++i) {
-      if (k[i] >= tk && k[i] > kth) {
+      if (k[i] >= tk && k[i] > thr) {
         c[3] = c[2];
         c[2] = c[1];
         c[1] = c[0];
@@ -243,6 +304,12 @@ topk_marginals_kernel(const T* __restrict__ logits, int64_t row_stride, int V, i
       }
     }
     const bool wide = __any_sync(kFullMask, cnt > 4);
+    // the tile's top-KP lies among these candidates: when they are few, insert
+    // them rather than run KP rounds of a warp maximum
+    if (!wide && __reduce_add_sync(kFullMask, static_cast<unsigned>(cnt)) <= 2 * kFewKeys) {
+      insert_all(c, cnt);
+      return;
+    }
     uint64_t nrun = 0;
 #pragma unroll 1
     for (int r = 0; r < KP; ++r) {
@@ -269,6 +336,7 @@ topk_marginals_kernel(const T* __restrict__ logits, int64_t row_stride, int V, i
     }
     run = nrun;
     kth = __shfl_sync(kFullMask, nrun, KP - 1);
+    if (lane == 0 && kth > thr) atomicMax(&s_thr, static_cast<unsigned long long>(kth));
   };
 
   if (vec_ok) {
@@ -278,38 +346,78 @@ topk_marginals_kernel(const T* __restrict__ logits, int64_t row_stride, int V, i
     const int v0 = chunk * per;
     const int v1 = min(nvec, v0 + per);
     const uint4* xv = reinterpret_cast<const uint4*>(x);
-    for (int base = v0 + tid; base - tid < v1; base += 2 * kThreads) {
-      uint4 buf[2];
+    // Each thread streams its own next kRing - 1 tiles into a private ring
+    // in shared memory with 16-byte asynchronous copies (one commit group per
+    // tile), so that many tiles are in flight without holding registers; it
+    // reads back only what it copied itself, so no barrier is needed.
+    // Ring layout [slot][vector u][thread]: a warp's reads are contiguous.
+    constexpr int kStep = 2 * kThreads;
+    const uint32_t ring = static_cast<uint32_t>(__cvta_generic_to_shared(dyn_smem));
+    auto slot_addr = [&](int slot, int u) {
+      return ring + static_cast<uint32_t>(((slot * 2 + u) * kThreads + tid) * 16);
+    };
+    auto issue = [&](int slot, int base) {
 #pragma unroll
       for (int u = 0; u < 2; ++u) {
         const int v = base + u * kThreads;
-        if (v < v1) buf[u] = __ldcs(xv + v);
+        if (v < v1)
+          asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(slot_addr(slot, u)),
+                       "l"(xv + v)
+                       : "memory");
       }
-      uint64_t k[EPT];
+      asm volatile("cp.async.commit_group;" ::: "memory");
+    };
+#pragma unroll
+    for (int a = 0; a < kRing - 1; ++a) issue(a, v0 + tid + a * kStep);
+    int slot = 0;
+    for (int base = v0 + tid; base - tid < v1; base += kStep) {
+      issue((slot + kRing - 1) % kRing, base + (kRing - 1) * kStep);
+      asm volatile("cp.async.wait_group %0;" ::"n"(kRing - 1) : "memory");
+      uint4 buf[2];
+#pragma unroll
+      for (int u = 0; u < 2; ++u)
+        asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+                     : "=r"(buf[u].x), "=r"(buf[u].y), "=r"(buf[u].z), "=r"(buf[u].w)
+                     : "r"(slot_addr(slot, u)));
+      slot = slot + 1 == kRing ? 0 : slot + 1;
+      float vals[EPT];
+      bool live[2];
+      float tmax = -INFINITY;
 #pragma unroll
       for (int u = 0; u < 2; ++u) {
         const int v = base + u * kThreads;
         const T* e = reinterpret_cast<const T*>(&buf[u]);
-        if (v < v1) {
-          float vals[VE];
+        live[u] = v < v1;
+        if (live[u]) {
           float vmax = -INFINITY;
 #pragma unroll
           for (int i = 0; i < VE; ++i) {
-            vals[i] = to_f32<T>(e[i]);
-            vmax = fmaxf(vmax, vals[i]);
+            vals[u * VE + i] = to_f32<T>(e[i]);
+            vmax = fmaxf(vmax, vals[u * VE + i]);
           }
           stats_raise(st, vmax * kLog2e);
 #pragma unroll
-          for (int i = 0; i < VE; ++i) {
-            stats_add(st, vals[i] * kLog2e);
-            k[u * VE + i] = make_key(vals[i], static_cast<uint32_t>(v * VE + i));
-          }
-        } else {
-#pragma unroll
-          for (int i = 0; i < VE; ++i) k[u * VE + i] = 0;
+          for (int i = 0; i < VE; ++i) stats_add(st, vals[u * VE + i] * kLog2e);
+          tmax = fmaxf(tmax, vmax);
         }
       }
-      merge_tile(k);
+      // keys are built only for a tile holding a value at or above the current
+      // threshold's (a lower value has a lower key whatever its token id)
+      const uint64_t shared_thr = *reinterpret_cast<volatile unsigned long long*>(&s_thr);
+      const uint64_t thr = shared_thr > kth ? shared_thr : kth;
+      const float thr_v = thr ? ordered_to_f32(static_cast<uint32_t>(thr >> 32)) : -INFINITY;
+      if (__any_sync(kFullMask, (live[0] || live[1]) && (thr == 0 || tmax >= thr_v))) {
+        uint64_t k[EPT];
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+          const int v = base + u * kThreads;
+#pragma unroll
+          for (int i = 0; i < VE; ++i)
+            k[u * VE + i] =
+                live[u] ? make_key(vals[u * VE + i], static_cast<uint32_t>(v * VE + i)) : 0ull;
+        }
+        merge_tile(k);
+      }
     }
     // tail elements past the last full vector go to the last chunk
     if (chunk == chunks - 1 && nvec * VE < V) {
@@ -407,7 +515,16 @@ void launch(const void* logits, int64_t row_stride, const Plan& p, int V, int K,
   float4* st = p.chunks > 1 ? reinterpret_cast<float4*>(ws + w.stats) : nullptr;
   uint64_t* keys = p.chunks > 1 ? reinterpret_cast<uint64_t*>(ws + w.keys) : nullptr;
   unsigned* tk = p.chunks > 1 ? reinterpret_cast<unsigned*>(ws + w.tickets) : nullptr;
-  launch_dep(topk_marginals_kernel<KP, T>, grid, dim3(kThreads), 0, s,
+  // the copy ring exceeds the default 48 KB of dynamic shared memory: raise
+  // the limit once per device (setting it twice from racing threads is harmless)
+  static bool ring_attr[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) == cudaSuccess && dev >= 0 && dev < 64 && !ring_attr[dev]) {
+    cudaFuncSetAttribute(topk_marginals_kernel<KP, T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         static_cast<int>(kRingBytes));
+    ring_attr[dev] = true;
+  }
+  launch_dep(topk_marginals_kernel<KP, T>, grid, dim3(kThreads), vec_ok ? kRingBytes : 0, s,
              static_cast<const T*>(logits), row_stride, V, K, p.chunks, vec_ok, ids, logp, lse,
              ent, st, keys, tk);
 }
