@@ -16,9 +16,16 @@
 #include <mutex>
 
 #include "common.cuh"
+#include "sm100.cuh"
 
 namespace taps {
 namespace {
+
+using sm100::add_f32x2;
+using sm100::f32x2;
+using sm100::f32x2_split;
+using sm100::fma_f32x2;
+using sm100::mul_f32x2;
 
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
@@ -230,6 +237,19 @@ topk_marginals_kernel(const T* __restrict__ logits, int64_t row_stride, int V, i
   // and the running list; a lane with more than four (heavy ties) sends the
   // tile through the same rounds over all of its keys instead.
   constexpr int EPT = 2 * VE;
+  // Insert one key (the same in every lane, above the K-th or the list not
+  // full) into the lane-sorted running list: lane r < KP holds the r-th
+  // largest; the key goes to position pos = (entries above it) and the entries
+  // from pos on shift one lane down. A key that an earlier insertion has
+  // already pushed below the K-th (pos == KP) changes nothing.
+  auto insert_one = [&](uint64_t key) {
+    const int pos = __popc(__ballot_sync(kFullMask, lane < KP && run > key));
+    const uint64_t up = __shfl_up_sync(kFullMask, run, 1);
+    if (pos < KP) {
+      if (lane < KP && lane > pos) run = up;
+      if (lane == pos) run = key;
+    }
+  };
   auto merge_tile = [&](uint64_t (&k)[EPT]) {
     uint64_t lm = 0;
 #pragma unroll
@@ -250,15 +270,7 @@ topk_marginals_kernel(const T* __restrict__ logits, int64_t row_stride, int V, i
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
           if (j < n_src) {
-            const uint64_t key = __shfl_sync(kFullMask, c4[j], src);
-            const unsigned above = __ballot_sync(kFullMask, lane < KP && run > key);
-            const int pos = __popc(above);
-            const uint64_t up = __shfl_up_sync(kFullMask, run, 1);
-            // (an earlier insertion may have raised the K-th above this key)
-            if (pos < KP) {
-              if (lane < KP && lane > pos) run = up;
-              if (lane == pos) run = key;
-            }
+            insert_one(__shfl_sync(kFullMask, c4[j], src));
           }
         }
       }
@@ -352,6 +364,21 @@ topk_marginals_kernel(const T* __restrict__ logits, int64_t row_stride, int V, i
     // reads back only what it copied itself, so no barrier is needed.
     // Ring layout [slot][vector u][thread]: a warp's reads are contiguous.
     constexpr int kStep = 2 * kThreads;
+    // the statistics in packed pairs: two partial sums per thread (kept
+    // relative to the thread's running max st.m2), folded into st at the end
+    uint64_t zp = f32x2(0.f, 0.f), tp = f32x2(0.f, 0.f);
+    const uint64_t l2e = f32x2(kLog2e, kLog2e);
+    auto raise = [&](float m2_new) {
+      if (m2_new > st.m2) {
+        if (st.m2 > -INFINITY) {
+          const float dm = st.m2 - m2_new;
+          const uint64_t sc = f32x2(ex2f(dm), ex2f(dm));
+          tp = mul_f32x2(sc, fma_f32x2(zp, f32x2(dm, dm), tp));
+          zp = mul_f32x2(zp, sc);
+        }
+        st.m2 = m2_new;
+      }
+    };
     const uint32_t ring = static_cast<uint32_t>(__cvta_generic_to_shared(dyn_smem));
     auto slot_addr = [&](int slot, int u) {
       return ring + static_cast<uint32_t>(((slot * 2 + u) * kThreads + tid) * 16);
@@ -395,9 +422,22 @@ topk_marginals_kernel(const T* __restrict__ logits, int64_t row_stride, int V, i
             vals[u * VE + i] = to_f32<T>(e[i]);
             vmax = fmaxf(vmax, vals[u * VE + i]);
           }
-          stats_raise(st, vmax * kLog2e);
+          raise(vmax * kLog2e);
+          // per pair: d = x log2(e) - m2 (one rounding), clamped at -127 so
+          // that -inf and values far below the max give exactly 0 (ex2 with
+          // flush-to-zero) and never 0 * inf
+          const uint64_t nm2 = f32x2(-st.m2, -st.m2);
 #pragma unroll
-          for (int i = 0; i < VE; ++i) stats_add(st, vals[u * VE + i] * kLog2e);
+          for (int i = 0; i < VE; i += 2) {
+            float d0, d1;
+            f32x2_split(fma_f32x2(f32x2(vals[u * VE + i], vals[u * VE + i + 1]), l2e, nm2), d0,
+                        d1);
+            d0 = fmaxf(d0, -127.f);
+            d1 = fmaxf(d1, -127.f);
+            const uint64_t e = f32x2(ex2f(d0), ex2f(d1));
+            zp = add_f32x2(zp, e);
+            tp = fma_f32x2(e, f32x2(d0, d1), tp);
+          }
           tmax = fmaxf(tmax, vmax);
         }
       }
@@ -407,17 +447,53 @@ topk_marginals_kernel(const T* __restrict__ logits, int64_t row_stride, int V, i
       const uint64_t thr = shared_thr > kth ? shared_thr : kth;
       const float thr_v = thr ? ordered_to_f32(static_cast<uint32_t>(thr >> 32)) : -INFINITY;
       if (__any_sync(kFullMask, (live[0] || live[1]) && (thr == 0 || tmax >= thr_v))) {
-        uint64_t k[EPT];
+        // elements whose value reaches the threshold's value: only they can
+        // hold a key above it
+        uint32_t flag = 0;
 #pragma unroll
-        for (int u = 0; u < 2; ++u) {
-          const int v = base + u * kThreads;
+        for (int i = 0; i < EPT; ++i)
+          flag |= (live[i / VE] && vals[i] >= thr_v) ? (1u << i) : 0u;
+        const int nflag = __popc(flag);
+        if (thr != 0 && __reduce_add_sync(kFullMask, static_cast<unsigned>(nflag)) <= kFewKeys) {
+          // few: visit only the element slots some lane flagged, build those
+          // keys, and insert the ones above the threshold
 #pragma unroll
-          for (int i = 0; i < VE; ++i)
-            k[u * VE + i] =
-                live[u] ? make_key(vals[u * VE + i], static_cast<uint32_t>(v * VE + i)) : 0ull;
+          for (int i = 0; i < EPT; ++i) {
+            if (__any_sync(kFullMask, (flag >> i) & 1u)) {
+              const int v = base + (i / VE) * kThreads;
+              const uint64_t key =
+                  ((flag >> i) & 1u) ? make_key(vals[i], static_cast<uint32_t>(v * VE + i % VE))
+                                     : 0ull;
+              unsigned who = __ballot_sync(kFullMask, key > thr);
+              while (who) {
+                const int src = __ffs(who) - 1;
+                who &= who - 1;
+                insert_one(__shfl_sync(kFullMask, key, src));
+              }
+            }
+          }
+          kth = __shfl_sync(kFullMask, run, KP - 1);
+          if (lane == 0 && kth > thr) atomicMax(&s_thr, static_cast<unsigned long long>(kth));
+        } else {
+          uint64_t k[EPT];
+#pragma unroll
+          for (int u = 0; u < 2; ++u) {
+            const int v = base + u * kThreads;
+#pragma unroll
+            for (int i = 0; i < VE; ++i)
+              k[u * VE + i] =
+                  live[u] ? make_key(vals[u * VE + i], static_cast<uint32_t>(v * VE + i)) : 0ull;
+          }
+          merge_tile(k);
         }
-        merge_tile(k);
       }
+    }
+    {
+      float z0, z1, t0, t1;
+      f32x2_split(zp, z0, z1);
+      f32x2_split(tp, t0, t1);
+      st.z += z0 + z1;
+      st.t2 += t0 + t1;
     }
     // tail elements past the last full vector go to the last chunk
     if (chunk == chunks - 1 && nvec * VE < V) {
