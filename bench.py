@@ -579,6 +579,32 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
+def run_only_topk(args):
+    """Stage 1 alone on the workload's logits (for profiling it at a given batch
+    without allocating the KV caches): prints microseconds per call."""
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    import paper_2606_00487_gb300 as taps
+    import workloads as W
+    cfg = workload_config(args.workload, args.n_max, args.layers, args.mode)
+    ldt = torch.bfloat16 if cfg.logits_dtype == "bf16" else torch.float32
+    x = torch.from_numpy(W.make_logits(cfg)).to("cuda").to(ldt)
+    for _ in range(args.warmup):
+        taps.taps_topk_marginals(x, cfg.K)
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(args.steps):
+        taps.taps_topk_marginals(x, cfg.K)
+    b.record()
+    torch.cuda.synchronize()
+    us = a.elapsed_time(b) / args.steps * 1e3
+    nbytes = x.numel() * x.element_size()
+    print(json.dumps({"stage": "topk_marginals", "workload": cfg.name, "us_per_call": round(us, 2),
+                      "bytes": nbytes, "gbs": round(nbytes / us / 1e3, 1)}), flush=True)
+
+
 def run_reference(args):
     """The oracle arm: rank 0 times the CPU oracle; other ranks exit."""
     rank = int(os.environ.get("RANK", "0"))
@@ -624,6 +650,8 @@ def main():
                     choices=["taps", "no_scorer", "budget_fill", "ddtree"],
                     help="selection preset: TAPS, or one of its ablations")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--only-topk", action="store_true",
+                    help="time stage 1 alone on the workload's logits (profiling aid)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-child", action="store_true", help=argparse.SUPPRESS)
     args = ap.parse_args()
@@ -631,6 +659,8 @@ def main():
         args.warmup = 3
     if args.cpu_child:
         cpu_child(args)
+    elif args.only_topk:
+        run_only_topk(args)
     elif args.impl == "reference":
         run_reference(args)
     else:
