@@ -95,6 +95,24 @@ def test_topk_ties_and_minus_inf(taps):
     _check_topk(taps, x, 1)
 
 
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
+def test_topk_value_ties_at_the_threshold(taps, dtype):
+    """Long rows whose largest values repeat (quantised to a coarse grid), so
+    that the running threshold's value is shared by many elements and the
+    token-id tie-break decides membership: exercises the value pre-filter and
+    the insertion merges over many tiles and across the CTA's warps."""
+    rng = np.random.default_rng(17)
+    B, L, V = 4, 16, 151936
+    x = np.round(rng.standard_normal((B, L, V)) * 2.0 * 4) / 4        # steps of 0.25
+    for b in range(B):
+        for d in range(L):
+            top = rng.choice(V, size=20, replace=False)              # 20 tied maxima
+            x[b, d, top] = x[b, d].max() + 0.25
+    x = x.astype(np.float32)
+    _check_topk(taps, x, 8, dtype)
+    _check_topk(taps, x, 16, dtype)
+
+
 def test_topk_strided_rows(taps):
     """Rows with a stride that is not a multiple of 16 bytes take the scalar path."""
     rng = np.random.default_rng(4)
