@@ -451,6 +451,10 @@ def run_ours(args):
         "s5_attention_one_layer": lambda: r.verify_layer(q0, k0, v0, b0, ctx, outs[0]),
         "s6_accept": lambda: r.accept(target),
     }
+    # the latency-bound stages back to back in one graph (what a round spends
+    # outside top-K and verification)
+    stage_fns["s2_s3_s4_s6_in_one_graph"] = lambda: [stage_fns[k]() for k in (
+        "s2_score", "s3_select", "s4_mask", "s6_accept")]
     stage_us = {}
     for name, fn in stage_fns.items():
         g = torch.cuda.CUDAGraph()
