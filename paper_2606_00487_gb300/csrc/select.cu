@@ -1,26 +1,44 @@
 // Stage 3 of a TAPS round (Sec. 4.2-4.3, Eq. 2, Eq. 3, Algorithm 1):
 // reach, utility and the greedy budgeted prefix-closed selection.
 //
-// One warp per request, everything in shared memory. Algorithm 1 adds, one
-// node at a time, the unselected node of largest utility. Utility never
-// increases from a parent to a child (q_cond <= 1, den(d) non-decreasing,
-// monotone rounding) and ties favour the lower depth, so that node is always
-// a child of a selected node, and its ancestors are already selected. Among
-// the children of one selected node, they are selected in key order, so the
-// frontier only needs, per selected node, its best unselected child: when a
-// child of node p is taken, p's next child in key order (the largest key
-// below the taken one) enters the frontier, and the new node's best child
-// enters too. The frontier therefore never exceeds n_max + 1 entries. A step
-// is one 64-bit warp maximum over the frontier (held in registers), then lane
-// k computes child k of the new node and child k of its parent side by side,
-// and two more warp maxima pick the two entries.
+// Algorithm 1 adds, one node at a time, the unselected node of largest
+// utility. Utility never increases from a parent to a child (q_cond <= 1,
+// den(d) non-decreasing, monotone rounding) and ties favour the lower depth,
+// so under the total order of the selection key below every child ranks
+// strictly after its parent. The greedy loop therefore takes nodes in
+// descending key order, and its result is the set of the n_max largest keys
+// of the whole candidate tree (those with utility > tau), listed in key
+// order; a child's parent index is its parent's position in that list.
 //
-// Frontier key (larger = taken first): utility bits (non-negative floats
+// One CTA per request computes that set level-synchronously instead of one
+// node per step. It keeps T, the best n_max nodes found so far in key order,
+// and repeats a pass:
+//   1. list the members of T whose children have not been generated yet
+//      (in position order; at most 512 / K of them per pass);
+//   2. generate their children, one thread per child, and keep the ones
+//      that would enter T (utility > tau and, once T is full, a key above
+//      T's last key);
+//   3. rank T and the kept children together by counting, write the best
+//      n_max in order into the other buffer and renumber parent indices.
+// It stops when a pass generates every remaining child and keeps none. A
+// node that left T never returns (T's last key only rises once T is full),
+// and a child that was not kept ranks below every member of T; at the stop
+// all members have been expanded, so T is the n_max largest keys. The number
+// of passes is about the depth of the selected tree plus one.
+//
+// Selection key (larger = taken first): utility bits (non-negative floats
 // order like their bit patterns) | (31 - depth) | (2^18 - 1 - token) |
 // (511 - parent index), i.e. utility desc, depth asc, token asc, parent asc.
+// A key is compared only with keys whose parent indices refer to the same T,
+// and the relative order of two members of T never changes, so comparing
+// indices into the current T is the same as comparing final indices. Equal
+// keys (only possible with repeated token ids in a top-K row) are ordered by
+// their index in the ranked array, which keeps ranks a permutation.
 //
 // All reach/utility arithmetic is IEEE f32 round-to-nearest (explicit _rn
-// intrinsics, no contraction), root to leaf.
+// intrinsics, no contraction), root to leaf. q_cond is staged clamped to
+// [0, 1] (NaN to 0), which changes nothing for valid input and keeps every
+// child after its parent for any input.
 #include <algorithm>
 
 #include "common.cuh"
@@ -35,77 +53,89 @@ __device__ __forceinline__ uint64_t node_key(float util, int depth, int token, i
          static_cast<uint64_t>(511 - parent);
 }
 
-struct SelSmem {
-  float* q;          // [L][K][K]
-  int* ids;          // [L][K]
-  float* den;        // [32]
-  int* parent;       // [n_max]
-  float* reach;      // [n_max]
-  float* util;       // [n_max]
-  unsigned char* depth;   // [n_max]
-  unsigned char* slot;    // [n_max]
+constexpr int kThreads = 512;
+constexpr int kWarps = kThreads / 32;
+// children generated per pass (one per thread)
+constexpr int kCap = kThreads;
+// every pass expands at least one member of T, and a node enters T at most
+// once; this bound is never reached and only keeps the loop finite
+constexpr int kMaxPasses = 1 << 14;
+
+// One buffer of ranked nodes: T in [0, nT), kept children appended after it.
+struct NodeBuf {
+  uint64_t* key;
+  float* reach;
+  float* util;
+  int16_t* ppos;          // parent index into the same buffer (-1: root)
+  unsigned char* depth;
+  unsigned char* slot;    // top-K slot of the node's position
+  unsigned char* done;    // children already generated
 };
 
+struct SelSmem {
+  float* q;          // [L][K][K], clamped to [0, 1]
+  int* ids;          // [L][K]
+  float* den;        // [32]
+  char* buf0;        // two node buffers of n_max + kCap entries
+  char* buf1;
+  int16_t* newpos;   // [n_max] new index of each member of T (-1: dropped)
+  int16_t* list;     // [n_max] members to expand this pass
+  int* warp_cnt;     // [kWarps]
+  int* kept;         // [2] kept-children counters, alternating by pass
+};
+
+__host__ __device__ inline size_t sel_round16(size_t x) { return (x + 15) / 16 * 16; }
+
+__host__ __device__ inline size_t node_buf_bytes(size_t C) {
+  return sel_round16(8 * C) + 2 * sel_round16(4 * C) + sel_round16(2 * C) + 3 * sel_round16(C);
+}
+
+__device__ __forceinline__ NodeBuf node_buf(char* p, size_t C) {
+  NodeBuf nb;
+  nb.key = reinterpret_cast<uint64_t*>(p);       p += sel_round16(8 * C);
+  nb.reach = reinterpret_cast<float*>(p);        p += sel_round16(4 * C);
+  nb.util = reinterpret_cast<float*>(p);         p += sel_round16(4 * C);
+  nb.ppos = reinterpret_cast<int16_t*>(p);       p += sel_round16(2 * C);
+  nb.depth = reinterpret_cast<unsigned char*>(p); p += sel_round16(C);
+  nb.slot = reinterpret_cast<unsigned char*>(p); p += sel_round16(C);
+  nb.done = reinterpret_cast<unsigned char*>(p);
+  return nb;
+}
+
 __host__ __device__ inline size_t sel_smem_bytes(int L, int K, int n_max) {
+  const size_t C = static_cast<size_t>(n_max) + kCap;
   size_t o = 0;
-  o += sizeof(float) * L * K * K;
-  o += sizeof(int) * L * K;
-  o += sizeof(float) * 32;
-  o += sizeof(int) * n_max + 2 * sizeof(float) * n_max;
-  o += 2 * n_max;
-  return (o + 15) / 16 * 16;
+  o += sel_round16(sizeof(float) * L * K * K);
+  o += sel_round16(sizeof(int) * L * K);
+  o += sel_round16(sizeof(float) * 32);
+  o += 2 * node_buf_bytes(C);
+  o += 2 * sel_round16(2 * static_cast<size_t>(n_max));
+  o += sel_round16(sizeof(int) * kWarps) + sel_round16(sizeof(int) * 2);
+  return o;
 }
 
 __device__ SelSmem carve(char* base, int L, int K, int n_max) {
-  SelSmem s;
+  const size_t C = static_cast<size_t>(n_max) + kCap;
   char* p = base;
-  s.q = reinterpret_cast<float*>(p);        p += sizeof(float) * L * K * K;
-  s.ids = reinterpret_cast<int*>(p);        p += sizeof(int) * L * K;
-  s.den = reinterpret_cast<float*>(p);      p += sizeof(float) * 32;
-  s.parent = reinterpret_cast<int*>(p);     p += sizeof(int) * n_max;
-  s.reach = reinterpret_cast<float*>(p);    p += sizeof(float) * n_max;
-  s.util = reinterpret_cast<float*>(p);     p += sizeof(float) * n_max;
-  s.depth = reinterpret_cast<unsigned char*>(p); p += n_max;
-  s.slot = reinterpret_cast<unsigned char*>(p);
+  auto take = [&](size_t bytes) {
+    char* r = p;
+    p += sel_round16(bytes);
+    return r;
+  };
+  SelSmem s;
+  s.q = reinterpret_cast<float*>(take(sizeof(float) * L * K * K));
+  s.ids = reinterpret_cast<int*>(take(sizeof(int) * L * K));
+  s.den = reinterpret_cast<float*>(take(sizeof(float) * 32));
+  s.buf0 = take(node_buf_bytes(C));
+  s.buf1 = take(node_buf_bytes(C));
+  s.newpos = reinterpret_cast<int16_t*>(take(2 * static_cast<size_t>(n_max)));
+  s.list = reinterpret_cast<int16_t*>(take(2 * static_cast<size_t>(n_max)));
+  s.warp_cnt = reinterpret_cast<int*>(take(sizeof(int) * kWarps));
+  s.kept = reinterpret_cast<int*>(take(sizeof(int) * 2));
   return s;
 }
 
-// A frontier entry stands for the best unselected child of a selected node p:
-// its key, its reach, p's reach, and packed p (9 bits) | the child's slot (5)
-// | p's depth (5) | p's slot (5).
-__device__ __forceinline__ uint32_t pack_info(int p, int slot, int dp, int pslot) {
-  return (static_cast<uint32_t>(p) << 15) | (static_cast<uint32_t>(slot) << 10) |
-         (static_cast<uint32_t>(dp) << 5) | static_cast<uint32_t>(pslot);
-}
-
-// Key and reach of the child in slot j of a node at depth dp, row `row` of the
-// q_cond table (its own slot; 0 for the root), reach rp, selection index p.
-__device__ __forceinline__ uint64_t child_key(const SelSmem& s, int K, int dp, int row, int j,
-                                              float rp, int p, float& r) {
-  r = __fmul_rn(rp, s.q[(dp * K + row) * K + j]);
-  const float u = __fdiv_rn(r, s.den[dp + 1]);
-  return node_key(u, dp + 1, s.ids[dp * K + j], p);
-}
-
-// Frontier slot f lives in lane f % 32, entry f / 32 of that lane's arrays
-// (fully unrolled, so that the arrays stay in registers).
-template <int SPL>
-__device__ __forceinline__ void set_entry(uint64_t (&fk)[SPL], uint32_t (&fi)[SPL],
-                                          float (&fr)[SPL], float (&frp)[SPL], int lane, int f,
-                                          uint64_t key, uint32_t info, float r, float rp) {
-#pragma unroll
-  for (int i = 0; i < SPL; ++i) {
-    const bool hit = lane == (f & 31) && i == (f >> 5);
-    fk[i] = hit ? key : fk[i];
-    fi[i] = hit ? info : fi[i];
-    fr[i] = hit ? r : fr[i];
-    frp[i] = hit ? rp : frp[i];
-  }
-}
-
-// SPL: frontier slots per lane.
-template <int SPL>
-__global__ void __launch_bounds__(32)
+__global__ void __launch_bounds__(kThreads, 1)
 select_kernel(const float* __restrict__ q_cond, const int* __restrict__ ids,
               const int32_t* __restrict__ root_tok, const int32_t* __restrict__ ctx_len, int L,
               int K, float lambda1, float lambda2, float tau, int n_max,
@@ -116,146 +146,175 @@ select_kernel(const float* __restrict__ q_cond, const int* __restrict__ ids,
   dep_enter();
   extern __shared__ __align__(16) char smem_raw[];
   const int b = blockIdx.x;
-  const int lane = threadIdx.x;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   SelSmem s = carve(smem_raw, L, K, n_max);
+  const size_t C = static_cast<size_t>(n_max) + kCap;
 
   const float* qb = q_cond + static_cast<int64_t>(b) * L * K * K;
-  for (int i = lane; i < L * K * K; i += 32) s.q[i] = qb[i];
+  for (int i = tid; i < L * K * K; i += kThreads) {
+    const float v = qb[i];
+    s.q[i] = v > 0.f ? fminf(v, 1.0f) : 0.f;
+  }
   const int32_t* ib = ids + static_cast<int64_t>(b) * L * K;
-  for (int i = lane; i < L * K; i += 32) s.ids[i] = ib[i];
-  if (lane <= L) s.den[lane] = __fadd_rn(lambda1, __fmul_rn(lambda2, static_cast<float>(lane)));
-  if (lane == 0) {
-    s.parent[0] = -1;
-    s.depth[0] = 0;
-    s.slot[0] = 0;
-    s.reach[0] = 1.0f;
+  for (int i = tid; i < L * K; i += kThreads) s.ids[i] = ib[i];
+  if (tid <= L) s.den[tid] = __fadd_rn(lambda1, __fmul_rn(lambda2, static_cast<float>(tid)));
+  if (tid == 0) {
+    const float den0 = __fadd_rn(lambda1, __fmul_rn(lambda2, 0.0f));
+    NodeBuf T = node_buf(s.buf0, C);
+    T.key[0] = ~0ull;   // the root ranks first
+    T.reach[0] = 1.0f;
+    T.util[0] = __fdiv_rn(1.0f, den0);
+    T.ppos[0] = -1;
+    T.depth[0] = 0;
+    T.slot[0] = 0;
+    T.done[0] = 0;
+    s.kept[0] = 0;
   }
-  __syncwarp();
-  if (lane == 0) s.util[0] = __fdiv_rn(1.0f, s.den[0]);
+  __syncthreads();
 
-  // the frontier, in registers
-  uint64_t fk[SPL];
-  uint32_t fi[SPL];
-  float fr[SPL], frp[SPL];
-#pragma unroll
-  for (int i = 0; i < SPL; ++i) {
-    fk[i] = 0;
-    fi[i] = 0;
-    fr[i] = 0.f;
-    frp[i] = 0.f;
-  }
-  uint64_t my_best = 0;
-  int n = 1, fsize = 0;
+  const int max_expand = kCap / K;
+  int cur = 0, nT = 1;
+  for (int pass = 0; pass < kMaxPasses; ++pass) {
+    const NodeBuf T = node_buf(cur ? s.buf1 : s.buf0, C);
+    const NodeBuf Nx = node_buf(cur ? s.buf0 : s.buf1, C);
+    int* kept = s.kept + (pass & 1);
 
-  if (n < n_max && L > 0) {
-    float r = 0.f;
-    const uint64_t key = lane < K ? child_key(s, K, 0, 0, lane, 1.0f, 0, r) : 0ull;
-    const uint64_t k0 = warp_max_u64(key);
-    const int src = __ffs(__ballot_sync(kFullMask, key == k0)) - 1;
-    set_entry<SPL>(fk, fi, fr, frp, lane, 0, k0, pack_info(0, src, 0, 0),
-                   __shfl_sync(kFullMask, r, src), 1.0f);
-    fsize = 1;
-    my_best = lane == 0 ? fk[0] : 0ull;
-  }
-
-  while (n < n_max) {
-    const uint64_t best = warp_max_u64(my_best);
-    if (best == 0) break;
-    const float bu = __uint_as_float(static_cast<uint32_t>(best >> 32));
-    if (!(bu > tau)) break;
-    // the owner of the winning entry hands it to the warp
-    const int wl = __ffs(__ballot_sync(kFullMask, my_best == best)) - 1;
-    int wi = 0;
-    uint32_t info = 0;
-    float r = 0.f, rp = 0.f;
-#pragma unroll
-    for (int i = 0; i < SPL; ++i)
-      if (fk[i] == best) {
-        wi = i;
-        info = fi[i];
-        r = fr[i];
-        rp = frp[i];
-      }
-    const int fslot = (__shfl_sync(kFullMask, wi, wl) << 5) | wl;
-    info = __shfl_sync(kFullMask, info, wl);
-    r = __shfl_sync(kFullMask, r, wl);
-    rp = __shfl_sync(kFullMask, rp, wl);
-    const int p = static_cast<int>(info >> 15), j = static_cast<int>((info >> 10) & 31u);
-    const int dp = static_cast<int>((info >> 5) & 31u), pslot = static_cast<int>(info & 31u);
-    const int v = n, dv = dp + 1;
-    if (lane == 0) {
-      s.parent[v] = p;
-      s.depth[v] = static_cast<unsigned char>(dv);
-      s.slot[v] = static_cast<unsigned char>(j);
-      s.reach[v] = r;
-      s.util[v] = bu;
-    }
-    n++;
-    // child k of v and child k of p, side by side: in lanes k and K + k when
-    // 2K lanes suffice (one instruction stream: a divergent branch per node
-    // would run the two halves one after the other), else in two passes
-    const bool has_child = dv < L && n < n_max;
-    float rc = 0.f, rs = 0.f;
-    uint64_t kc = 0, ks = 0;
-    const int prow = dp == 0 ? 0 : pslot;
-    if (2 * K <= 32) {
-      const bool of_v = lane < K;
-      const int k = of_v ? lane : lane - K;
-      float rr = 0.f;
-      uint64_t key = 0;
-      if ((of_v && has_child) || (!of_v && k < K))
-        key = child_key(s, K, of_v ? dv : dp, of_v ? j : prow, k, of_v ? r : rp, of_v ? v : p, rr);
-      if (of_v) {
-        kc = key;
-        rc = rr;
-      } else {
-        ks = key < best ? key : 0ull;   // p's children taken so far have keys >= the popped one
-        rs = rr;
-      }
-    } else {
-      if (lane < K && has_child) kc = child_key(s, K, dv, j, lane, r, v, rc);
-      if (lane < K) {
-        ks = child_key(s, K, dp, prow, lane, rp, p, rs);
-        if (ks >= best) ks = 0;
+    // 1. members still to expand, in position order
+    const bool open = tid < nT && !T.done[tid];
+    const unsigned bal = __ballot_sync(kFullMask, open);
+    if (lane == 0) s.warp_cnt[warp] = __popc(bal);
+    __syncthreads();
+    // the other counter was last read before this barrier
+    if (tid == 0) s.kept[(pass + 1) & 1] = 0;
+    const int wc = lane < kWarps ? s.warp_cnt[lane] : 0;
+    const int before = __reduce_add_sync(kFullMask, lane < warp ? wc : 0);
+    const int total = __reduce_add_sync(kFullMask, wc);
+    const int X = min(total, max_expand);
+    if (open) {
+      const int idx = before + __popc(bal & ((1u << lane) - 1u));
+      if (idx < X) {
+        s.list[idx] = static_cast<int16_t>(tid);
+        T.done[tid] = 1;
       }
     }
-    const uint64_t k0 = warp_max_u64(kc);
-    const uint64_t k1 = warp_max_u64(ks);
-    const int c0 = k0 ? __ffs(__ballot_sync(kFullMask, kc == k0)) - 1 : 0;
-    const int l1 = k1 ? __ffs(__ballot_sync(kFullMask, ks == k1)) - 1 : 0;
-    const int c1 = 2 * K <= 32 && k1 ? l1 - K : l1;   // the child slot of p's entry
-    const float r0 = __shfl_sync(kFullMask, rc, c0);
-    const float r1 = __shfl_sync(kFullMask, rs, l1);
-    // the popped slot takes the sibling (else the child), a fresh slot the child
-    const uint32_t child_info = pack_info(v, c0, dv, j);
-    if (k1) {
-      set_entry<SPL>(fk, fi, fr, frp, lane, fslot, k1, pack_info(p, c1, dp, pslot), r1, rp);
-      if (k0) {
-        set_entry<SPL>(fk, fi, fr, frp, lane, fsize, k0, child_info, r0, r);
-        fsize++;
-      }
-    } else {
-      set_entry<SPL>(fk, fi, fr, frp, lane, fslot, k0, child_info, r0, r);
-    }
-    my_best = 0;
-#pragma unroll
-    for (int i = 0; i < SPL; ++i) my_best = fk[i] > my_best ? fk[i] : my_best;
-  }
-  __syncwarp();
+    __syncthreads();
 
-  // write the selected nodes in selection order, pad the rest
+    // 2. their children; keep those that would enter T
+    const uint64_t thr = nT == n_max ? T.key[nT - 1] : 0ull;
+    bool keep = false;
+    uint64_t key = 0;
+    float r = 0.f, u = 0.f;
+    int t = 0, j = 0, dc = 0;
+    if (tid < X * K) {
+      const int li = tid / K;
+      j = tid - li * K;
+      t = s.list[li];
+      const int dp = T.depth[t];
+      dc = dp + 1;
+      const int row = dp == 0 ? 0 : T.slot[t];
+      r = __fmul_rn(T.reach[t], s.q[(dp * K + row) * K + j]);
+      u = __fdiv_rn(r, s.den[dc]);
+      key = node_key(u, dc, s.ids[dp * K + j], t);
+      keep = u > tau && key > thr;
+    }
+    const unsigned kb = __ballot_sync(kFullMask, keep);
+    int base = 0;
+    if (lane == 0 && kb) base = atomicAdd(kept, __popc(kb));
+    base = __shfl_sync(kFullMask, base, 0);
+    if (keep) {
+      const int e = nT + base + __popc(kb & ((1u << lane) - 1u));
+      T.key[e] = key;
+      T.reach[e] = r;
+      T.util[e] = u;
+      T.ppos[e] = static_cast<int16_t>(t);
+      T.depth[e] = static_cast<unsigned char>(dc);
+      T.slot[e] = static_cast<unsigned char>(j);
+      T.done[e] = dc >= L;
+    }
+    __syncthreads();
+    const int m = *kept;
+    if (m == 0) {
+      if (total == X) break;
+      continue;
+    }
+
+    // 3. rank T and the kept children: g threads per entry
+    const int E = nT + m;
+    int lg = 5;
+    while (lg > 0 && (E << lg) > kThreads) --lg;
+    const int g = 1 << lg;
+    const int grp = tid >> lg, sub = tid & (g - 1);
+    for (int e0 = 0; e0 < E; e0 += kThreads >> lg) {
+      const int e = e0 + grp;
+      int cnt = 0;
+      uint64_t ke = 0;
+      if (e < E) {
+        ke = T.key[e];
+        if (e < nT) {
+          // members ahead of it: e; children ahead of it: those of larger key
+          if (sub == 0) cnt = e;
+          for (int c = nT + sub; c < E; c += g) cnt += T.key[c] > ke ? 1 : 0;
+        } else {
+          // members with key >= ke: a prefix of T (its keys descend)
+          if (sub == 0) {
+            int lo = 0, hi = nT;
+            while (lo < hi) {
+              const int mid = (lo + hi) >> 1;
+              if (T.key[mid] >= ke) lo = mid + 1;
+              else hi = mid;
+            }
+            cnt = lo;
+          }
+          for (int c = nT + sub; c < E; c += g) {
+            const uint64_t kc = T.key[c];
+            cnt += (c < e ? kc >= ke : kc > ke) ? 1 : 0;
+          }
+        }
+      }
+      for (int o = 1; o < g; o <<= 1) cnt += __shfl_xor_sync(kFullMask, cnt, o);
+      if (sub == 0 && e < E) {
+        if (e < nT) s.newpos[e] = static_cast<int16_t>(cnt < n_max ? cnt : -1);
+        if (cnt < n_max) {
+          Nx.key[cnt] = ke;
+          Nx.reach[cnt] = T.reach[e];
+          Nx.util[cnt] = T.util[e];
+          Nx.ppos[cnt] = T.ppos[e];
+          Nx.depth[cnt] = T.depth[e];
+          Nx.slot[cnt] = T.slot[e];
+          Nx.done[cnt] = T.done[e];
+        }
+      }
+    }
+    __syncthreads();
+    // renumber parents (a parent always ranks before its child, so it stayed)
+    nT = min(E, n_max);
+    if (tid < nT) {
+      const int po = Nx.ppos[tid];
+      if (po >= 0) {
+        const int pn = s.newpos[po];
+        Nx.ppos[tid] = static_cast<int16_t>(pn);
+        Nx.key[tid] = (Nx.key[tid] & ~511ull) | static_cast<uint64_t>(511 - pn);
+      }
+    }
+    cur ^= 1;
+    // the next pass reads these entries only after its first barrier
+  }
+  __syncthreads();
+
+  // write the selected nodes in key order, pad the rest
+  const NodeBuf T = node_buf(cur ? s.buf1 : s.buf0, C);
   const int64_t o = static_cast<int64_t>(b) * n_max;
   const int c = ctx_len[b];
-  for (int i = lane; i < n_max; i += 32) {
-    if (i < n) {
-      int d = s.depth[i];
-      parent_out[o + i] = s.parent[i];
+  for (int i = tid; i < n_max; i += kThreads) {
+    if (i < nT) {
+      const int d = T.depth[i];
+      parent_out[o + i] = T.ppos[i];
       depth_out[o + i] = d;
-      slot_out[o + i] = i == 0 ? -1 : s.slot[i];
-      token_out[o + i] = i == 0 ? root_tok[b] : s.ids[(d - 1) * K + s.slot[i]];
+      slot_out[o + i] = i == 0 ? -1 : T.slot[i];
+      token_out[o + i] = i == 0 ? root_tok[b] : s.ids[(d - 1) * K + T.slot[i]];
       pos_out[o + i] = c + d;
-      reach_out[o + i] = s.reach[i];
-      util_out[o + i] = s.util[i];
+      reach_out[o + i] = T.reach[i];
+      util_out[o + i] = T.util[i];
     } else {
       parent_out[o + i] = -1;
       depth_out[o + i] = -1;
@@ -266,10 +325,9 @@ select_kernel(const float* __restrict__ q_cond, const int* __restrict__ ids,
       util_out[o + i] = 0.f;
     }
   }
-  if (lane == 0) n_nodes_out[b] = n;
+  if (tid == 0) n_nodes_out[b] = nT;
 }
 
-template <int SPL>
 int launch_select(const float* q_cond, const int32_t* topk_ids, const int32_t* root_tok,
                   const int32_t* ctx_len, int B, int L, int K, float l1, float l2, float tau,
                   int n_max, int32_t* n_nodes, int32_t* parent, int32_t* depth, int32_t* token,
@@ -277,12 +335,12 @@ int launch_select(const float* q_cond, const int32_t* topk_ids, const int32_t* r
                   cudaStream_t stream) {
   const size_t smem = sel_smem_bytes(L, K, n_max);
   if (smem > 48 * 1024 &&
-      cudaFuncSetAttribute(select_kernel<SPL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+      cudaFuncSetAttribute(select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            static_cast<int>(smem)) != cudaSuccess)
     return TAPS_ERR_CUDA;
-  if (launch_dep(select_kernel<SPL>, dim3(B), dim3(32), smem, stream, q_cond, topk_ids, root_tok,
-                 ctx_len, L, K, l1, l2, tau, n_max, n_nodes, parent, depth, token, slot, pos_id,
-                 reach, utility) != cudaSuccess)
+  if (launch_dep(select_kernel, dim3(B), dim3(kThreads), smem, stream, q_cond, topk_ids,
+                 root_tok, ctx_len, L, K, l1, l2, tau, n_max, n_nodes, parent, depth, token,
+                 slot, pos_id, reach, utility) != cudaSuccess)
     return TAPS_ERR_CUDA;
   return launch_status();
 }
@@ -306,15 +364,7 @@ extern "C" int taps_select_subtree(const float* q_cond, const int32_t* topk_ids,
   if (!(l1 > 0.f) || !(l2 >= 0.f) || !(tau >= 0.f) || n_max < 1) return TAPS_ERR_INVALID_ARG;
   if (K > TAPS_MAX_K || L > TAPS_MAX_L || n_max > TAPS_MAX_NODES || B > 65535)
     return TAPS_ERR_UNSUPPORTED;
-  // the frontier holds at most one entry per selected node (n_max + 1)
-  const int fmax = n_max + 1;
-  cudaStream_t st = static_cast<cudaStream_t>(stream);
-#define TAPS_SELECT_LAUNCH(SPL)                                                               \
-  return launch_select<SPL>(q_cond, topk_ids, root_tok, ctx_len, B, L, K, l1, l2, tau, n_max, \
-                            n_nodes, parent, depth, token, slot, pos_id, reach, utility, st)
-  if (fmax <= 32) TAPS_SELECT_LAUNCH(1);
-  if (fmax <= 96) TAPS_SELECT_LAUNCH(3);
-  if (fmax <= 288) TAPS_SELECT_LAUNCH(9);
-  TAPS_SELECT_LAUNCH(17);
-#undef TAPS_SELECT_LAUNCH
+  return launch_select(q_cond, topk_ids, root_tok, ctx_len, B, L, K, l1, l2, tau, n_max,
+                       n_nodes, parent, depth, token, slot, pos_id, reach, utility,
+                       static_cast<cudaStream_t>(stream));
 }
