@@ -54,7 +54,6 @@ __device__ __forceinline__ uint64_t node_key(float util, int depth, int token, i
 }
 
 constexpr int kThreads = 512;
-constexpr int kWarps = kThreads / 32;
 // children generated per pass (one per thread)
 constexpr int kCap = kThreads;
 // every pass expands at least one member of T, and a node enters T at most
@@ -79,9 +78,12 @@ struct SelSmem {
   char* buf0;        // two node buffers of n_max + kCap entries
   char* buf1;
   int16_t* newpos;   // [n_max] new index of each member of T (-1: dropped)
-  int16_t* list;     // [n_max] members to expand this pass
-  int* warp_cnt;     // [kWarps]
-  int* kept;         // [2] kept-children counters, alternating by pass
+  int16_t* list;     // [n_max] members to expand this pass, with their
+  float* lreach;     //   reach,
+  unsigned char* ldepth;  // depth and q_cond row
+  unsigned char* lrow;
+  int* cnt;          // [4] listed-member and kept-child counters, two each,
+                     //     alternating by pass
 };
 
 __host__ __device__ inline size_t sel_round16(size_t x) { return (x + 15) / 16 * 16; }
@@ -109,8 +111,8 @@ __host__ __device__ inline size_t sel_smem_bytes(int L, int K, int n_max) {
   o += sel_round16(sizeof(int) * L * K);
   o += sel_round16(sizeof(float) * 32);
   o += 2 * node_buf_bytes(C);
-  o += 2 * sel_round16(2 * static_cast<size_t>(n_max));
-  o += sel_round16(sizeof(int) * kWarps) + sel_round16(sizeof(int) * 2);
+  o += 2 * sel_round16(2 * static_cast<size_t>(n_max)) + sel_round16(4 * static_cast<size_t>(n_max));
+  o += 2 * sel_round16(static_cast<size_t>(n_max)) + sel_round16(sizeof(int) * 4);
   return o;
 }
 
@@ -130,9 +132,28 @@ __device__ SelSmem carve(char* base, int L, int K, int n_max) {
   s.buf1 = take(node_buf_bytes(C));
   s.newpos = reinterpret_cast<int16_t*>(take(2 * static_cast<size_t>(n_max)));
   s.list = reinterpret_cast<int16_t*>(take(2 * static_cast<size_t>(n_max)));
-  s.warp_cnt = reinterpret_cast<int*>(take(sizeof(int) * kWarps));
-  s.kept = reinterpret_cast<int*>(take(sizeof(int) * 2));
+  s.lreach = reinterpret_cast<float*>(take(4 * static_cast<size_t>(n_max)));
+  s.ldepth = reinterpret_cast<unsigned char*>(take(static_cast<size_t>(n_max)));
+  s.lrow = reinterpret_cast<unsigned char*>(take(static_cast<size_t>(n_max)));
+  s.cnt = reinterpret_cast<int*>(take(sizeof(int) * 4));
   return s;
+}
+
+// Number of keys above k among key[c0], key[c0 + g], ... below index hi;
+// eight independent loads in flight.
+__device__ __forceinline__ int count_above(const uint64_t* key, int c0, int hi, int g,
+                                           uint64_t k) {
+  int cnt = 0;
+  int c = c0;
+  for (; c + 7 * g < hi; c += 8 * g) {
+    uint64_t v[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) v[i] = key[c + i * g];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) cnt += v[i] > k ? 1 : 0;
+  }
+  for (; c < hi; c += g) cnt += key[c] > k ? 1 : 0;
+  return cnt;
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
@@ -146,7 +167,7 @@ select_kernel(const float* __restrict__ q_cond, const int* __restrict__ ids,
   dep_enter();
   extern __shared__ __align__(16) char smem_raw[];
   const int b = blockIdx.x;
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int tid = threadIdx.x, lane = tid & 31;
   SelSmem s = carve(smem_raw, L, K, n_max);
   const size_t C = static_cast<size_t>(n_max) + kCap;
 
@@ -168,53 +189,63 @@ select_kernel(const float* __restrict__ q_cond, const int* __restrict__ ids,
     T.depth[0] = 0;
     T.slot[0] = 0;
     T.done[0] = 0;
-    s.kept[0] = 0;
+    s.cnt[0] = 0;
+    s.cnt[2] = 0;
   }
   __syncthreads();
 
   const int max_expand = kCap / K;
+  // this thread's child in step 2: child j_own of listed member li_own
+  const int li_own = tid / K;
+  const int j_own = tid - li_own * K;
   int cur = 0, nT = 1;
   for (int pass = 0; pass < kMaxPasses; ++pass) {
     const NodeBuf T = node_buf(cur ? s.buf1 : s.buf0, C);
     const NodeBuf Nx = node_buf(cur ? s.buf0 : s.buf1, C);
-    int* kept = s.kept + (pass & 1);
+    int* listed = s.cnt + (pass & 1);
+    int* kept = s.cnt + 2 + (pass & 1);
 
-    // 1. members still to expand, in position order
+    // 1. list members still to expand (any order); the first max_expand
+    //    listed are expanded in this pass, the rest in a later one
     const bool open = tid < nT && !T.done[tid];
     const unsigned bal = __ballot_sync(kFullMask, open);
-    if (lane == 0) s.warp_cnt[warp] = __popc(bal);
-    __syncthreads();
-    // the other counter was last read before this barrier
-    if (tid == 0) s.kept[(pass + 1) & 1] = 0;
-    const int wc = lane < kWarps ? s.warp_cnt[lane] : 0;
-    const int before = __reduce_add_sync(kFullMask, lane < warp ? wc : 0);
-    const int total = __reduce_add_sync(kFullMask, wc);
-    const int X = min(total, max_expand);
+    int lbase = 0;
+    if (lane == 0 && bal) lbase = atomicAdd(listed, __popc(bal));
+    lbase = __shfl_sync(kFullMask, lbase, 0);
     if (open) {
-      const int idx = before + __popc(bal & ((1u << lane) - 1u));
-      if (idx < X) {
+      const int idx = lbase + __popc(bal & ((1u << lane) - 1u));
+      if (idx < max_expand) {
+        const int dp = T.depth[tid];
         s.list[idx] = static_cast<int16_t>(tid);
+        s.lreach[idx] = T.reach[tid];
+        s.ldepth[idx] = static_cast<unsigned char>(dp);
+        s.lrow[idx] = dp == 0 ? 0 : T.slot[tid];
         T.done[tid] = 1;
       }
     }
     __syncthreads();
+    // the other pair of counters was last read before this barrier
+    if (tid == 0) {
+      s.cnt[(pass + 1) & 1] = 0;
+      s.cnt[2 + ((pass + 1) & 1)] = 0;
+    }
+    const int total = *listed;
+    const int X = min(total, max_expand);
 
     // 2. their children; keep those that would enter T
     const uint64_t thr = nT == n_max ? T.key[nT - 1] : 0ull;
     bool keep = false;
     uint64_t key = 0;
     float r = 0.f, u = 0.f;
-    int t = 0, j = 0, dc = 0;
-    if (tid < X * K) {
-      const int li = tid / K;
-      j = tid - li * K;
-      t = s.list[li];
-      const int dp = T.depth[t];
+    int t = 0, dc = 0;
+    if (li_own < X) {
+      t = s.list[li_own];
+      const int dp = s.ldepth[li_own];
+      const int row = s.lrow[li_own];
       dc = dp + 1;
-      const int row = dp == 0 ? 0 : T.slot[t];
-      r = __fmul_rn(T.reach[t], s.q[(dp * K + row) * K + j]);
+      r = __fmul_rn(s.lreach[li_own], s.q[(dp * K + row) * K + j_own]);
       u = __fdiv_rn(r, s.den[dc]);
-      key = node_key(u, dc, s.ids[dp * K + j], t);
+      key = node_key(u, dc, s.ids[dp * K + j_own], t);
       keep = u > tau && key > thr;
     }
     const unsigned kb = __ballot_sync(kFullMask, keep);
@@ -228,7 +259,7 @@ select_kernel(const float* __restrict__ q_cond, const int* __restrict__ ids,
       T.util[e] = u;
       T.ppos[e] = static_cast<int16_t>(t);
       T.depth[e] = static_cast<unsigned char>(dc);
-      T.slot[e] = static_cast<unsigned char>(j);
+      T.slot[e] = static_cast<unsigned char>(j_own);
       T.done[e] = dc >= L;
     }
     __syncthreads();
@@ -250,25 +281,37 @@ select_kernel(const float* __restrict__ q_cond, const int* __restrict__ ids,
       uint64_t ke = 0;
       if (e < E) {
         ke = T.key[e];
+        // entries ahead of e on this lane's stride, counted over up to three
+        // ranges with their thresholds (one loop, so that one copy of the
+        // counting code serves every case)
+        const uint64_t ke1 = ke - 1;   // kept keys are >= 2^32: "> ke1" is ">= ke"
+        const int c0 = nT + sub;
+        int lo0 = 0, hi0 = 0, split = c0;
         if (e < nT) {
-          // members ahead of it: e; children ahead of it: those of larger key
+          // a member: members ahead of it are e; children ahead have a larger key
           if (sub == 0) cnt = e;
-          for (int c = nT + sub; c < E; c += g) cnt += T.key[c] > ke ? 1 : 0;
         } else {
-          // members with key >= ke: a prefix of T (its keys descend)
-          if (sub == 0) {
-            int lo = 0, hi = nT;
+          // a kept child: members with key >= ke (a prefix of T, whose keys
+          // descend), then children with key >= ke before it and > ke after it
+          if (nT <= 32 * g) {
+            lo0 = sub;
+            hi0 = nT;
+          } else {
+            int lo = 0, hi = sub < nT ? ((nT - 1 - sub) >> lg) + 1 : 0;
             while (lo < hi) {
               const int mid = (lo + hi) >> 1;
-              if (T.key[mid] >= ke) lo = mid + 1;
+              if (T.key[sub + mid * g] > ke1) lo = mid + 1;
               else hi = mid;
             }
             cnt = lo;
           }
-          for (int c = nT + sub; c < E; c += g) {
-            const uint64_t kc = T.key[c];
-            cnt += (c < e ? kc >= ke : kc > ke) ? 1 : 0;
-          }
+          if (e > c0) split = c0 + (((e - c0 + g - 1) >> lg) << lg);
+        }
+#pragma unroll 1
+        for (int rg = 0; rg < 3; ++rg) {
+          const int lo = rg == 0 ? lo0 : rg == 1 ? c0 : split;
+          const int hi = rg == 0 ? hi0 : rg == 1 ? split : E;
+          cnt += count_above(T.key, lo, hi, g, rg == 2 ? ke : ke1);
         }
       }
       for (int o = 1; o < g; o <<= 1) cnt += __shfl_xor_sync(kFullMask, cnt, o);
