@@ -14,7 +14,7 @@
 // node per step. It keeps T, the best n_max nodes found so far in key order,
 // and repeats a pass:
 //   1. list the members of T whose children have not been generated yet
-//      (in position order; at most 512 / K of them per pass);
+//      (in any order; at most 512 / K of them per pass, the rest wait);
 //   2. generate their children, one thread per child, and keep the ones
 //      that would enter T (utility > tau and, once T is full, a key above
 //      T's last key);

@@ -334,6 +334,47 @@ def test_frontier_equals_literal_algorithm1(seed):
             _check_tree_invariants(s, 0, ids, 3, 10, n_max, L)
 
 
+@pytest.mark.parametrize("seed", range(12))
+def test_algorithm1_is_the_top_n_of_the_trie(seed):
+    """Algorithm 1 adds nodes in descending key order, so its result is the
+    n_max largest nodes of the whole trie (utility > tau) under the key order
+    utility desc, depth asc, token asc, then the parents' own order (Eq. 3 and
+    the argmax of Algorithm 1): a plain sort of the materialised trie must give
+    the same nodes in the same order. Half the cases carry exact utility ties."""
+    import functools
+    rng = np.random.default_rng(300 + seed)
+    L, K = [(3, 2), (2, 3), (4, 2), (3, 3)][seed % 4]
+    ties = seed % 2 == 1
+    q = _random_qcond(rng, L, K, ties)[None]
+    ids = np.stack([rng.permutation(20)[:K] for _ in range(L)]).astype(np.int32)[None]
+    lam2 = [0.0, 0.3, 0.1][seed % 3]
+    nodes = O.materialise_trie(q[0], ids[0], 3, 1.0, lam2, L, K)
+
+    def cmp(a, b):
+        if a == b:
+            return 0
+        ua, ub = float(nodes[a]["utility"]), float(nodes[b]["utility"])
+        if ua != ub:
+            return -1 if ua > ub else 1
+        if len(a) != len(b):
+            return -1 if len(a) < len(b) else 1
+        ta, tb = nodes[a]["token"], nodes[b]["token"]
+        if ta != tb:
+            return -1 if ta < tb else 1
+        return cmp(a[:-1], b[:-1])
+
+    for tau in (0.0, 0.05):
+        alive = [p for p in nodes if p == () or nodes[p]["utility"] > np.float32(tau)]
+        ranked = sorted(alive, key=functools.cmp_to_key(cmp))
+        for n_max in (1, 3, len(nodes) // 3, len(nodes)):
+            s = O.select_subtree(q, ids, np.array([3]), np.array([10]), 1.0, lam2, tau, n_max)
+            n = int(s["n_nodes"][0])
+            paths = [()]
+            for i in range(1, n):
+                paths.append(paths[int(s["parent"][0, i])] + (int(s["slot"][0, i]),))
+            assert paths == ranked[:n_max]
+
+
 def _prefix_closed_subsets(all_paths, size):
     nonroot = [p for p in all_paths if p != ()]
     for combo in itertools.combinations(nonroot, size - 1):
