@@ -1,6 +1,6 @@
 """Parity of every CUDA stage (through the C ABI) with the CPU oracle.
 
-Tolerances (derived in the design doc):
+Tolerances (each follows from the arithmetic of its stage):
 * integer results (top-K ids, tree topology, mask, acceptance) bit-exact;
 * lse, entropy: 1e-5 relative; logp = logit - lse: 1e-5 of max(|logp|, |lse|);
 * q_cond (same inputs on both sides): 1e-5 relative, 1e-7 absolute floor;
