@@ -13,6 +13,8 @@ notation, slowly and plainly:
 * ``score_qcond``      Sec. 4.2, Eq. 1 and Algorithm 1 (sibling softmax of
                        the scorer logits).
 * ``reach_of_path``    Sec. 4.2, Eq. 2 (product of q_cond along the path).
+* ``path_reach``       Eq. 2 for an explicit list of nodes, in the float32
+                       arithmetic that decides the tree.
 * ``select_subtree``   Sec. 4.3, Eq. 3 and Algorithm 1 (greedy budgeted
                        prefix-closed selection), argmax over the frontier.
 * ``select_subtree_literal``  Algorithm 1 over a fully materialised candidate
@@ -169,6 +171,36 @@ def reach_of_path(q_cond_b: np.ndarray, slots) -> float:
         r *= float(q_cond_b[d, parent_slot, j])
         parent_slot = j
     return r
+
+
+def path_reach(q_cond, paths, path_len):
+    """Eq. 2 for an explicit list of trie nodes, in the arithmetic that decides
+    the tree: q_reach = product of q_cond along root -> node, float32 with one
+    IEEE round-to-nearest multiply per edge, root to leaf (the same operations
+    and order as the reach in ``select_subtree``).
+
+    q_cond [B, L, K, K]; paths [B, M, L] top-K slots (a node at depth n is
+    named by the slots of its first n edges); path_len [B, M] in [0, L].
+    Returns [B, M] float32; a length of 0 is the root (reach 1). A node that
+    is not in the trie (length outside [0, L], or a slot >= K among its first
+    path_len entries) gets reach 0.
+    """
+    B, L, K, _ = q_cond.shape
+    M = paths.shape[1]
+    out = np.zeros((B, M), F32)
+    for b in range(B):
+        for m in range(M):
+            n = int(path_len[b, m])
+            slots = [int(j) for j in paths[b, m, :max(n, 0)]]
+            if n < 0 or n > L or any(j >= K for j in slots):
+                continue
+            r = F32(1.0)
+            parent_slot = 0                       # depth-1 children hang off the root (row 0)
+            for d, j in enumerate(slots):
+                r = F32(r * F32(q_cond[b, d, parent_slot, j]))
+                parent_slot = j
+            out[b, m] = r
+    return out
 
 
 # ---------------------------------------------------------------------------
@@ -441,30 +473,3 @@ def compact_accepted_kv(k_cache, v_cache, block_table, ctx_len, accepted_nodes, 
             k_new[dp, :, dr, :] = k_cache[sp, :, sr, :]
             v_new[dp, :, dr, :] = v_cache[sp, :, sr, :]
     return k_new, v_new
-
-
-# ---------------------------------------------------------------------------
-# A whole round (used by the CPU baseline and the end-to-end parity tests)
-# ---------------------------------------------------------------------------
-
-def run_round(logits, K, root_tok, ctx_len, select_params, scorer_kind, scorer_weights,
-              target_seq, layers):
-    """Stages 1-6 in the paper's order. ``layers`` is a list of
-    (q, k_cache, v_cache, block_table) tuples, one per verified layer;
-    ``target_seq`` gives the target's greedy continuation y (see workloads).
-    """
-    ids, logp, lse, ent = topk_marginals(logits, K)
-    q_cond = score_qcond(root_tok, ids, logp, ent, scorer_kind, scorer_weights)
-    sel = select_subtree(q_cond, ids, root_tok, ctx_len, **select_params)
-    n_max = select_params["n_max"]
-    mask = build_tree_mask(sel["parent"], sel["n_nodes"], n_max)
-    attn = [tree_verify_attn(q, kc, vc, bt, ctx_len, sel["n_nodes"], mask)
-            for (q, kc, vc, bt) in layers]
-    B = ids.shape[0]
-    target_tok = np.full((B, n_max), -1, np.int32)
-    for b in range(B):
-        n = int(sel["n_nodes"][b])
-        target_tok[b, :n] = target_seq[b, sel["depth"][b, :n]]
-    acc = accept(sel["parent"], sel["token"], sel["n_nodes"], target_tok, ids.shape[1])
-    return dict(ids=ids, logp=logp, lse=lse, entropy=ent, q_cond=q_cond, sel=sel, mask=mask,
-                attn=attn, target_tok=target_tok, accept=acc)

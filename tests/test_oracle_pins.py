@@ -427,6 +427,71 @@ def test_reach_is_product_of_qcond(seed):
         assert s["utility"][0, i] == pytest.approx(exact / den, rel=1e-6)
 
 
+def test_path_reach_hand_worked():
+    """Eq. 2 on a two-level trie whose q_cond values are exact in float32:
+    every product is exact, and a wrong parent row or a transposed q_cond
+    index changes the (1, 0) and (0, 1) entries."""
+    q = np.zeros((1, 2, 2, 2), F32)
+    q[0, 0, 0] = [0.75, 0.25]           # depth-1 children of the root (row 0)
+    q[0, 1, 0] = [0.5, 0.5]             # children of slot 0
+    q[0, 1, 1] = [0.125, 0.875]         # children of slot 1
+    cases = {(): 1.0, (0,): 0.75, (1,): 0.25, (0, 0): 0.375, (0, 1): 0.375,
+             (1, 0): 0.03125, (1, 1): 0.21875}
+    paths = np.zeros((1, len(cases) + 3, 2), np.uint8)
+    plen = np.zeros((1, len(cases) + 3), np.int32)
+    for m, path in enumerate(cases):
+        paths[0, m, :len(path)] = path
+        plen[0, m] = len(path)
+    m0 = len(cases)
+    paths[0, m0] = [2, 0]; plen[0, m0] = 1            # slot 2 >= K: not a node
+    paths[0, m0 + 1] = [0, 0]; plen[0, m0 + 1] = 3    # deeper than L: not a node
+    paths[0, m0 + 2] = [1, 2]; plen[0, m0 + 2] = 1    # the bad slot lies past the length
+    r = O.path_reach(q, paths, plen)
+    assert r.dtype == F32
+    assert r[0, :m0].tolist() == list(cases.values())
+    assert r[0, m0:].tolist() == [0.0, 0.0, 0.25]
+
+
+@pytest.mark.parametrize("seed", range(3))
+def test_path_reach_within_rounding_of_exact_product(seed):
+    """float32, one rounding per edge: within L * 2^-24 (relative) of the
+    float64 product of the same q_cond values."""
+    rng = np.random.default_rng(500 + seed)
+    B, L, K, M = 2, 12, 5, 40
+    q = np.stack([_random_qcond(rng, L, K) for _ in range(B)])
+    paths = rng.integers(0, K, size=(B, M, L)).astype(np.uint8)
+    plen = rng.integers(0, L + 1, size=(B, M)).astype(np.int32)
+    r = O.path_reach(q, paths, plen)
+    for b in range(B):
+        for m in range(M):
+            exact = O.reach_of_path(q[b].astype(np.float64), paths[b, m, :plen[b, m]].tolist())
+            assert abs(float(r[b, m]) - exact) <= L * 2.0 ** -24 * exact * 1.0001
+
+
+def test_path_reach_equals_the_selected_tree_reach():
+    """The reach that decides the tree (select_subtree, built parent to child)
+    and path_reach of each selected node's slot path are the same float32
+    operations in the same order: bit-identical."""
+    rng = np.random.default_rng(77)
+    B, L, K = 2, 7, 4
+    q = np.stack([_random_qcond(rng, L, K) for _ in range(B)])
+    ids = np.stack([np.stack([rng.permutation(100)[:K] for _ in range(L)])
+                    for _ in range(B)]).astype(np.int32)
+    s = O.select_subtree(q, ids, np.array([1, 2]), np.array([0, 0]), 1.0, 0.1, 0.0, 90)
+    paths = np.zeros((B, 90, L), np.uint8)
+    plen = np.zeros((B, 90), np.int32)
+    for b in range(B):
+        walk = [()]
+        for i in range(1, int(s["n_nodes"][b])):
+            walk.append(walk[int(s["parent"][b, i])] + (int(s["slot"][b, i]),))
+            paths[b, i, :len(walk[-1])] = walk[-1]
+            plen[b, i] = len(walk[-1])
+    r = O.path_reach(q, paths, plen)
+    for b in range(B):
+        n = int(s["n_nodes"][b])
+        assert r[b, :n].view(np.uint32).tolist() == s["reach"][b, :n].view(np.uint32).tolist()
+
+
 def test_children_reach_sums_to_parent_reach():
     rng = np.random.default_rng(7)
     L, K = 3, 3
