@@ -35,6 +35,7 @@ sys.path.insert(0, ROOT)
 
 FALLBACK_HBM_GBS = 6800.0
 FALLBACK_BF16_TFLOPS = 1900.0
+FALLBACK_BF16_TFLOPS_SUSTAINED = 1700.0
 
 
 def attn_source_sha256():
@@ -48,13 +49,18 @@ def attn_source_sha256():
 
 
 def load_peaks():
+    """(HBM GB/s, bf16 TF/s burst, bf16 TF/s sustained, source). The attention
+    kernel runs inside a long step, so its tensor rate is compared with the
+    sustained figure."""
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
         with open(p) as f:
             d = json.load(f)
-        return float(d["hbm_gbs"]), float(d["bf16_tflops"]), "measured"
+        burst = float(d["bf16_tflops"])
+        return (float(d["hbm_gbs"]), burst, float(d.get("bf16_tflops_sustained", burst)),
+                "measured")
     except Exception:
-        return FALLBACK_HBM_GBS, FALLBACK_BF16_TFLOPS, "fallback"
+        return FALLBACK_HBM_GBS, FALLBACK_BF16_TFLOPS, FALLBACK_BF16_TFLOPS_SUSTAINED, "fallback"
 
 
 # scorer kind and (lambda2, tau) overrides of each selection preset; the
@@ -141,10 +147,11 @@ class ClockSampler:
 # CPU baseline: the oracle as it stands, on a bounded sample of the workload
 # ---------------------------------------------------------------------------
 
-def oracle_step(cfg, inp, sample_layers, kind="mlp"):
+def oracle_step(cfg, inp, sample_layers, kind="mlp", pool=None):
     """One oracle round: stages 1-4 and 6 on the whole batch, stage 5 on
     ``sample_layers`` of the cfg.layers layers; returns seconds scaled to the
-    full round."""
+    full round. With ``pool`` (worker processes holding the same inputs), each
+    sampled layer's stage 5 is split over the workers by (request, head)."""
     from oracle import taps_oracle as O
     t0 = time.perf_counter()
     ids, logp, lse, ent = O.topk_marginals(inp["logits"], cfg.K)
@@ -156,10 +163,20 @@ def oracle_step(cfg, inp, sample_layers, kind="mlp"):
     tt = W.target_tokens_for_tree(inp["y"], sel["depth"], sel["n_nodes"])
     O.accept(sel["parent"], sel["token"], sel["n_nodes"], tt, cfg.L)
     t1 = time.perf_counter()
-    for _ in range(sample_layers):
-        O.tree_verify_attn(inp["q"], inp["k"], inp["v"], inp["bt"], inp["ctx"], sel["n_nodes"],
-                           mask)
-    t2 = time.perf_counter()
+    if pool is not None:
+        # each task: a group of (request, head) pairs and this round's tree
+        n_w = pool._processes
+        pairs = [(b, h) for b in range(cfg.B) for h in range(cfg.Hq)]
+        tasks = [(pairs[i::n_w], sel["n_nodes"], mask) for i in range(n_w)]
+        for _ in range(sample_layers):
+            # the workers' outputs cover disjoint rows: their sum is the layer's output
+            sum(pool.map(_attn_worker_rows, tasks, chunksize=1))
+        t2 = time.perf_counter()
+    else:
+        for _ in range(sample_layers):
+            O.tree_verify_attn(inp["q"], inp["k"], inp["v"], inp["bt"], inp["ctx"],
+                               sel["n_nodes"], mask)
+        t2 = time.perf_counter()
     per_layer = (t2 - t1) / max(sample_layers, 1)
     return (t1 - t0) + cfg.layers * per_layer, t2 - t0
 
@@ -167,38 +184,81 @@ def oracle_step(cfg, inp, sample_layers, kind="mlp"):
 def oracle_inputs(cfg):
     import workloads as W
     logits = W.make_logits(cfg)
+    inp = oracle_attn_inputs(cfg)
+    inp.update(logits=logits, root=W.make_root_tokens(cfg), w=W.make_scorer_weights(cfg),
+               y=W.make_target_sequence(cfg, logits))
+    return inp
+
+
+def oracle_attn_inputs(cfg):
+    import workloads as W
     ctx = W.make_ctx_lens(cfg)
     bt, num_pages = W.make_block_table(cfg, ctx)
     k, v = W.make_kv_numpy(cfg, num_pages)
-    return dict(logits=logits, root=W.make_root_tokens(cfg), ctx=ctx, bt=bt, k=k, v=v,
-                q=W.make_q_numpy(cfg, cfg.B, cfg.n_max), w=W.make_scorer_weights(cfg),
-                y=W.make_target_sequence(cfg, logits))
+    return dict(ctx=ctx, bt=bt, k=k, v=v, q=W.make_q_numpy(cfg, cfg.B, cfg.n_max))
+
+
+# worker-process state of the all-cores oracle (spawned processes, no CUDA)
+_W = {}
+
+
+def _attn_worker_init(cfg):
+    # one BLAS thread per worker process (numpy is first imported below)
+    for v in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+        os.environ[v] = "1"
+    _W["cfg"] = cfg
+    _W["inp"] = oracle_attn_inputs(cfg)
+
+
+def _attn_worker_ready(_):
+    return "inp" in _W
+
+
+def _attn_worker_rows(task):
+    """Stage 5 of the oracle for the given (request, head) pairs, every node."""
+    from oracle import taps_oracle as O
+    pairs, nn, mask = task
+    inp = _W["inp"]
+    only = {(b, i, h) for (b, h) in pairs for i in range(int(nn[b]))}
+    out, _ = O.tree_verify_attn(inp["q"], inp["k"], inp["v"], inp["bt"], inp["ctx"], nn, mask,
+                                only=only)
+    return out
 
 
 def cpu_child(args):
-    """Runs in a fresh single-threaded process: prints the oracle timing JSON."""
+    """Runs in a fresh process without CUDA: prints the oracle timing JSON."""
     cfg = workload_config(args.workload, args.n_max, args.layers, args.mode)
     kind = MODE_PARAMS[args.mode][0]
     inp = oracle_inputs(cfg)
+    pool = None
+    if args.cpu_cores > 1:
+        import multiprocessing as mp
+        pool = mp.get_context("spawn").Pool(args.cpu_cores, initializer=_attn_worker_init,
+                                            initargs=(cfg,))
+        assert all(pool.map(_attn_worker_ready, range(4 * args.cpu_cores), chunksize=1))
     steps, warm = args.steps, args.warmup
     for _ in range(warm):
-        oracle_step(cfg, inp, args.sample_layers, kind)
+        oracle_step(cfg, inp, args.sample_layers, kind, pool)
     scaled, wall = [], []
     for _ in range(steps):
-        s, w = oracle_step(cfg, inp, args.sample_layers, kind)
+        s, w = oracle_step(cfg, inp, args.sample_layers, kind, pool)
         scaled.append(s)
         wall.append(w)
-    print(json.dumps({"scaled_s": scaled, "wall_s": wall}))
+    if pool is not None:
+        pool.close()
+        pool.join()
+    print(json.dumps({"scaled_s": scaled, "wall_s": wall, "cores": args.cpu_cores}))
 
 
-def run_cpu_baseline(args, steps, warmup, sample_layers):
+def run_cpu_baseline(args, steps, warmup, sample_layers, cores=1):
     cfg = workload_config(args.workload, args.n_max, args.layers, args.mode)
     env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1",
                CUDA_VISIBLE_DEVICES="")
     cmd = [sys.executable, os.path.abspath(__file__), "--cpu-child", "--workload", args.workload,
            "--mode", args.mode,
            "--n-max", str(cfg.n_max), "--layers", str(cfg.layers), "--steps", str(steps),
-           "--warmup", str(warmup), "--sample-layers", str(sample_layers)]
+           "--warmup", str(warmup), "--sample-layers", str(sample_layers),
+           "--cpu-cores", str(cores)]
     r = subprocess.run(cmd, env=env, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"cpu baseline child failed:\n{r.stderr[-2000:]}")
@@ -295,7 +355,7 @@ def after_verify(taps, W, cfg, r, layers, bt, ctx, target, sel_h, s, stream, rep
     assert int(r.status.item()) == 0, "device fault status after compaction"
     live = int(sel_h["n_nodes"].sum())
     k7_bytes = live * cfg.V * 2
-    hbm, _, _ = load_peaks()
+    hbm = load_peaks()[0]
     gbs = k7_bytes / (k7_us * 1e-6) / 1e9
     moved = int(r.accept_len.sum().item()) + cfg.B
     del bufs
@@ -310,8 +370,165 @@ def after_verify(taps, W, cfg, r, layers, bt, ctx, target, sel_h, s, stream, rep
     }
 
 
+class RoundSetup:
+    """Every device buffer of one workload's round (seeded synthetic inputs,
+    KV caches and queries drawn on the device), the TapsRound and its three
+    CUDA graphs (stages 1-4, the per-layer attention calls, stage 6)."""
+
+    def __init__(self, taps, W, cfg, mode, dev):
+        import torch
+        self.cfg = cfg
+        self.logits_h = W.make_logits(cfg)
+        root_h, self.ctx_h = W.make_root_tokens(cfg), W.make_ctx_lens(cfg)
+        w = W.make_scorer_weights(cfg)
+        self.bt_h, num_pages = W.make_block_table(cfg, self.ctx_h)
+        self.y = W.make_target_sequence(cfg, self.logits_h)
+        ldt = torch.bfloat16 if cfg.logits_dtype == "bf16" else torch.float32
+        # the round's per-step inputs live in one staging buffer (one upload per round)
+        self.inp = inp = taps.RoundInputs(B=cfg.B, L=cfg.L, V=cfg.V, n_max=cfg.n_max, Hq=cfg.Hq,
+                                          D=cfg.D, layers=cfg.layers, logits_dtype=ldt,
+                                          device=dev)
+        self.logits = inp.dev["logits"]
+        self.logits.copy_(torch.from_numpy(self.logits_h).to(dev).to(ldt))
+        self.root = inp.dev["root_tok"]
+        self.root.copy_(torch.from_numpy(root_h).to(dev))
+        self.ctx = torch.from_numpy(self.ctx_h).to(dev)
+        self.bt = torch.from_numpy(self.bt_h).to(dev)
+        self.layers = []
+        for layer in range(cfg.layers):
+            kc, vc = W.make_kv_torch(cfg, num_pages, layer, dev)
+            kc, vc = taps.taps_pack_kv_pages(kc), taps.taps_pack_kv_pages(vc)   # TAPS page layout
+            q = inp.dev["q"][layer]
+            q.copy_(W.make_q_torch(cfg, cfg.B, cfg.n_max, layer, dev))
+            self.layers.append((q, kc, vc, self.bt))
+        self.outs = [torch.empty_like(self.layers[0][0]) for _ in range(cfg.layers)]
+        self.r = r = taps.TapsRound(
+            B=cfg.B, L=cfg.L, V=cfg.V, K=cfg.K, n_max=cfg.n_max, Hq=cfg.Hq, Hkv=cfg.Hkv,
+            D=cfg.D, max_ctx=int(self.ctx_h.max()), device=dev,
+            scorer_weights=torch.from_numpy(w["packed"]).to(dev), emb_dim=w["E"], hidden=w["H"],
+            lambda1=cfg.lambda1, lambda2=cfg.lambda2, tau=cfg.tau,
+            mode=None if mode == "taps" else mode)
+        assert (r.lambda2, r.tau) == (cfg.lambda2, cfg.tau)
+        # the stand-in target model's greedy tokens depend on the (deterministic) tree
+        r.select(self.logits, self.root, self.ctx)
+        torch.cuda.synchronize()
+        self.sel_h = {k: v.cpu().numpy() for k, v in r.sel.items()}
+        tt_h = W.target_tokens_for_tree(self.y, self.sel_h["depth"], self.sel_h["n_nodes"])
+        self.target = inp.dev["target_tok"]
+        self.target.copy_(torch.from_numpy(tt_h).to(dev))
+        self.kv_bytes = sum(kc.numel() * kc.element_size() + vc.numel() * vc.element_size()
+                            for (_, kc, vc, _) in self.layers)
+
+        # ---- capture the round as three graphs
+        self.s = s = torch.cuda.Stream(device=dev)
+        s.wait_stream(torch.cuda.current_stream(dev))
+        with torch.cuda.stream(s):
+            for _ in range(2):
+                r.run(self.logits, self.root, self.ctx, self.layers, self.outs, self.target)
+        torch.cuda.current_stream(dev).wait_stream(s)
+        torch.cuda.synchronize()
+        self.g_pre, self.g_attn, self.g_post = (torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph(),
+                                                torch.cuda.CUDAGraph())
+        with torch.cuda.graph(self.g_pre, stream=s):
+            r.select(self.logits, self.root, self.ctx)
+        with torch.cuda.graph(self.g_attn, stream=s):
+            for (q, kc, vc, b_t), o in zip(self.layers, self.outs):
+                r.verify_layer(q, kc, vc, b_t, self.ctx, o)
+        with torch.cuda.graph(self.g_post, stream=s):
+            r.accept(self.target)
+        torch.cuda.synchronize()
+        self.stream = torch.cuda.current_stream(dev)
+
+    def step(self, ev_a=None, ev_b=None):
+        self.g_pre.replay()
+        if ev_a is not None:
+            ev_a.record(self.stream)
+        self.g_attn.replay()
+        if ev_b is not None:
+            ev_b.record(self.stream)
+        self.g_post.replay()
+
+    def time_steps(self, steps, warmup, world=1, clocks=None):
+        """W untimed rounds, then exactly ``steps`` rounds between a barrier and
+        a synchronize on each side. Returns (elapsed ms of the whole region,
+        per-round ms, per-round attention ms), each round's and its attention
+        stage's span taken with CUDA events on the launching stream."""
+        import torch
+        for _ in range(warmup):
+            self.step()
+        torch.cuda.synchronize()
+        if clocks is not None:
+            clocks.start()
+            time.sleep(0.3)
+        ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(steps)]
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        barrier(world)
+        torch.cuda.synchronize()
+        e0.record(self.stream)
+        for k in range(steps):
+            ev[k][0].record(self.stream)
+            self.step(ev[k][1], ev[k][2])
+        e1.record(self.stream)
+        torch.cuda.synchronize()
+        barrier(world)
+        elapsed_ms = e0.elapsed_time(e1)
+        rounds = [ev[k][0].elapsed_time(ev[k + 1][0]) for k in range(steps - 1)]
+        rounds.append(ev[-1][0].elapsed_time(e1))
+        attn = [a.elapsed_time(b) for (_, a, b) in ev]
+        return elapsed_ms, rounds, attn
+
+    def roofline(self, attn_ms_per_round, peaks):
+        """Attention (the dominant kernel): algorithmic bytes and flops of one
+        layer over its average launch time, against the measured HBM copy rate
+        and the sustained bf16 tensor rate; ``bound`` is the roofline whose
+        floor is higher for this workload."""
+        hbm, _, bf16_sus, src = peaks
+        byt, fl = attn_bytes_flops(self.cfg, self.ctx_h, self.sel_h["n_nodes"],
+                                   self.sel_h["depth"])
+        per_launch_s = attn_ms_per_round / self.cfg.layers / 1e3
+        gbs = byt / per_launch_s / 1e9
+        tf = fl / per_launch_s / 1e12
+        t_hbm, t_tc = byt / (hbm * 1e9), fl / (bf16_sus * 1e12)
+        return {"bound": "hbm" if t_hbm >= t_tc else "tensor",
+                "achieved_gbs": round(gbs, 1), "hbm_frac": round(gbs / hbm, 4),
+                "tensor_tflops": round(tf, 1), "tensor_frac": round(tf / bf16_sus, 4),
+                "floor_us": round(max(t_hbm, t_tc) * 1e6, 2),
+                "avg_launch_us": round(per_launch_s * 1e6, 2),
+                "algorithmic_bytes_per_launch": byt, "algorithmic_flops_per_launch": fl,
+                "peak_source": src}
+
+
+# The other configurations of the benchmark suite: the node-budget sweep at
+# the Qwen3-8B shape, the Qwen3-4B shape, the batch-32 serving round and the
+# long-context stress round (workload name, node budget).
+SWEEP = [("qwen3_8b", 32), ("qwen3_8b", 128), ("qwen3_8b", 256), ("qwen3_4b", 64),
+         ("batched", 64), ("long", 256)]
+
+
+def run_sweep(taps, W, args, dev, peaks):
+    import torch
+    out = {}
+    steps, warmup = max(5, min(args.steps, 20)), 3
+    for name, n in SWEEP:
+        cfg = workload_config(name, n, None, args.mode)
+        rs = RoundSetup(taps, W, cfg, args.mode, dev)
+        elapsed_ms, rounds, attn = rs.time_steps(steps, warmup)
+        status = int(rs.r.status.item())
+        rl = rs.roofline(statistics.median(attn), peaks)
+        out[f"{name}_n{n}"] = {
+            "rounds_per_s": round(steps / (elapsed_ms / 1e3), 2),
+            "ms_per_round_median": round(statistics.median(rounds), 4),
+            "B": cfg.B, "n_max": n, "layers": cfg.layers,
+            "n_nodes_total": int(rs.sel_h["n_nodes"].sum()),
+            "attention": rl, "steps": steps, "device_status": status}
+        assert status == 0, f"device fault status {status} on {name}"
+        del rs
+        torch.cuda.synchronize()
+        torch.cuda.empty_cache()
+    return out
+
+
 def run_ours(args):
-    import numpy as np
     import torch
 
     import __graft_entry__
@@ -323,96 +540,16 @@ def run_ours(args):
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     cfg = workload_config(args.workload, args.n_max, args.layers, args.mode)
+    peaks = load_peaks()
 
-    # ---- inputs (seeded, synthetic; KV and Q drawn on the device)
-    logits_h = W.make_logits(cfg)
-    root_h, ctx_h = W.make_root_tokens(cfg), W.make_ctx_lens(cfg)
-    w = W.make_scorer_weights(cfg)
-    bt_h, num_pages = W.make_block_table(cfg, ctx_h)
-    y = W.make_target_sequence(cfg, logits_h)
-    ldt = torch.bfloat16 if cfg.logits_dtype == "bf16" else torch.float32
-    # the round's per-step inputs live in one staging buffer (one upload per round)
-    inp = taps.RoundInputs(B=cfg.B, L=cfg.L, V=cfg.V, n_max=cfg.n_max, Hq=cfg.Hq, D=cfg.D,
-                           layers=cfg.layers, logits_dtype=ldt, device=dev)
-    logits = inp.dev["logits"]
-    logits.copy_(torch.from_numpy(logits_h).to(dev).to(ldt))
-    root = inp.dev["root_tok"]
-    root.copy_(torch.from_numpy(root_h).to(dev))
-    ctx = torch.from_numpy(ctx_h).to(dev)
-    bt = torch.from_numpy(bt_h).to(dev)
-    layers = []
-    for layer in range(cfg.layers):
-        kc, vc = W.make_kv_torch(cfg, num_pages, layer, dev)
-        kc, vc = taps.taps_pack_kv_pages(kc), taps.taps_pack_kv_pages(vc)   # TAPS page layout
-        q = inp.dev["q"][layer]
-        q.copy_(W.make_q_torch(cfg, cfg.B, cfg.n_max, layer, dev))
-        layers.append((q, kc, vc, bt))
-    outs = [torch.empty_like(layers[0][0]) for _ in range(cfg.layers)]
-
-    r = taps.TapsRound(B=cfg.B, L=cfg.L, V=cfg.V, K=cfg.K, n_max=cfg.n_max, Hq=cfg.Hq,
-                       Hkv=cfg.Hkv, D=cfg.D, max_ctx=int(ctx_h.max()), device=dev,
-                       scorer_weights=torch.from_numpy(w["packed"]).to(dev), emb_dim=w["E"],
-                       hidden=w["H"], lambda1=cfg.lambda1, lambda2=cfg.lambda2, tau=cfg.tau,
-                       mode=None if args.mode == "taps" else args.mode)
-    assert (r.lambda2, r.tau) == (cfg.lambda2, cfg.tau)
-    # the stand-in target model's greedy tokens depend on the (deterministic) tree
-    r.select(logits, root, ctx)
-    torch.cuda.synchronize()
-    sel_h = {k: v.cpu().numpy() for k, v in r.sel.items()}
-    tt_h = W.target_tokens_for_tree(y, sel_h["depth"], sel_h["n_nodes"])
-    target = inp.dev["target_tok"]
-    target.copy_(torch.from_numpy(tt_h).to(dev))
-
-    # ---- capture the round as three graphs
-    s = torch.cuda.Stream(device=dev)
-    s.wait_stream(torch.cuda.current_stream(dev))
-    with torch.cuda.stream(s):
-        for _ in range(2):
-            r.run(logits, root, ctx, layers, outs, target)
-    torch.cuda.current_stream(dev).wait_stream(s)
-    torch.cuda.synchronize()
-    g_pre, g_post = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
-    with torch.cuda.graph(g_pre, stream=s):
-        r.select(logits, root, ctx)
-    g_attn_all = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(g_attn_all, stream=s):
-        for (q, kc, vc, b_t), o in zip(layers, outs):
-            r.verify_layer(q, kc, vc, b_t, ctx, o)
-    with torch.cuda.graph(g_post, stream=s):
-        r.accept(target)
-    torch.cuda.synchronize()
-
-    stream = torch.cuda.current_stream(dev)
-
-    def step(ev_a=None, ev_b=None):
-        g_pre.replay()
-        if ev_a is not None:
-            ev_a.record(stream)
-        g_attn_all.replay()
-        if ev_b is not None:
-            ev_b.record(stream)
-        g_post.replay()
-
-    for _ in range(args.warmup):
-        step()
-    torch.cuda.synchronize()
+    rs = RoundSetup(taps, W, cfg, args.mode, dev)
+    r, s, stream = rs.r, rs.s, rs.stream
+    logits, root, ctx, target = rs.logits, rs.root, rs.ctx, rs.target
+    layers, outs, sel_h = rs.layers, rs.outs, rs.sel_h
 
     clocks = ClockSampler(local)
-    clocks.start()
-    time.sleep(0.3)
-    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-           for _ in range(args.steps)]
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    barrier(world)
-    torch.cuda.synchronize()
-    e0.record(stream)
-    for k in range(args.steps):
-        step(*evs[k])
-    e1.record(stream)
-    torch.cuda.synchronize()
-    barrier(world)
-    elapsed_ms = e0.elapsed_time(e1)
-    attn_ms = sum(a.elapsed_time(b) for a, b in evs) / args.steps
+    elapsed_ms, rounds_ms, attn_list = rs.time_steps(args.steps, args.warmup, world, clocks)
+    attn_ms = sum(attn_list) / args.steps
     clk = clocks.stop()
     elapsed_ms = max_over_ranks(elapsed_ms, world, dev)
     status = int(r.status.item())
@@ -429,7 +566,7 @@ def run_ours(args):
         g_one.replay()
     torch.cuda.synchronize()
     f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    reps = max(args.steps, 20)
+    reps = max(min(args.steps, 200), 20)
     f0.record(stream)
     for _ in range(reps):
         g_one.replay()
@@ -474,11 +611,13 @@ def run_ours(args):
     # greedy token per node fused with acceptance, and the accepted path's K/V
     # commit over all layers. The verify logits rotate over enough buffers to
     # exceed L2, so every launch reads its logits from HBM.
-    after = after_verify(taps, W, cfg, r, layers, bt, ctx, target, sel_h, s, stream, reps, dev)
+    after = after_verify(taps, W, cfg, r, layers, rs.bt, ctx, target, sel_h, s, stream, reps,
+                         dev)
     stage_us.update(after.pop("stage_us"))
 
     # ---- end to end through the public API with host buffers
     e2e = None
+    inp = rs.inp
     if not args.no_e2e:
         # the host staging buffer holds every input of a round (logits, root
         # tokens, the 36 layers' tree queries, target tokens): one upload per
@@ -499,10 +638,10 @@ def run_ours(args):
             inp.upload_head(stream)
             inp.upload_queries(copy_stream)
             q_ready.record(copy_stream)
-            g_pre.replay()
+            rs.g_pre.replay()
             stream.wait_event(q_ready)
-            g_attn_all.replay()
-            g_post.replay()
+            rs.g_attn.replay()
+            rs.g_post.replay()
             r.download(res_pin, stream)
             stream.synchronize()
 
@@ -514,15 +653,12 @@ def run_ours(args):
         for _ in range(args.steps):
             e2e_step()
         t_e2e = max_over_ranks(time.perf_counter() - t0, world, dev)
-        e2e = {"value": world * args.steps / t_e2e, "unit": "rounds/s",
+        e2e = {"value": round(world * args.steps / t_e2e, 2), "unit": "rounds/s",
                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}
 
     # ---- roofline of the attention stage (dominant kernel)
-    hbm, bf16, src = load_peaks()
-    byt, fl = attn_bytes_flops(cfg, ctx_h, sel_h["n_nodes"], sel_h["depth"])
-    per_launch_s = attn_ms / cfg.layers / 1e3
-    achieved_gbs = byt / per_launch_s / 1e9
-    achieved_tf = fl / per_launch_s / 1e12
+    hbm, bf16_burst, bf16_sus, src = peaks
+    rl = rs.roofline(attn_ms, peaks)
     traffic = None
     tp = os.path.join(ROOT, "profiles", "attn_traffic.json")
     if os.path.exists(tp):
@@ -534,31 +670,38 @@ def run_ours(args):
                 traffic = t.get("bytes_per_launch")
         except Exception:
             traffic = None
-    roofline = {"bound": "hbm", "achieved": round(achieved_gbs, 1), "peak": hbm, "unit": "GB/s",
-                "frac": round(achieved_gbs / hbm, 4), "traffic": traffic,
+    roofline = {"bound": "hbm", "achieved": rl["achieved_gbs"], "peak": hbm, "unit": "GB/s",
+                "frac": rl["hbm_frac"], "traffic": traffic,
                 "peak_source": src, "kernel": "taps_tree_verify_attn (one layer)",
-                "algorithmic_bytes_per_launch": byt, "avg_launch_us": round(per_launch_s * 1e6, 2),
-                "tensor_tflops": round(achieved_tf, 1),
-                "tensor_frac": round(achieved_tf / bf16, 4)}
+                "algorithmic_bytes_per_launch": rl["algorithmic_bytes_per_launch"],
+                "avg_launch_us": rl["avg_launch_us"],
+                "tensor_tflops": rl["tensor_tflops"], "tensor_frac": rl["tensor_frac"],
+                "tensor_peak": bf16_sus,
+                "tensor_peak_note": "sustained bf16 (the kernel runs inside a long step)",
+                "binding_roofline": rl["bound"], "floor_us": rl["floor_us"]}
+
+    sweep = None
+    if not args.no_sweep and args.workload == "qwen3_8b" and args.n_max in (None, 64):
+        sweep = run_sweep(taps, W, args, dev, peaks)
 
     launches = args.steps * (r.launches_per_select + cfg.layers * r.launches_per_layer + 1)
-    kv_bytes = sum(kc.numel() * kc.element_size() + vc.numel() * vc.element_size()
-                   for (_, kc, vc, _) in layers)
     line = {
         "metric": metric_name(args.workload),
         "value": round(world * args.steps / (elapsed_ms / 1e3), 2),
         "unit": "rounds/s",
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": round(elapsed_ms / args.steps, 4),
+        "ms_per_step_median": round(statistics.median(rounds_ms), 4),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": f"synthetic (seeded; shapes of the {SHAPE_NAMES.get(args.workload, args.workload)} "
                 "round, no weights or datasets)",
         "config": {"workload": f"{cfg.name}: B={cfg.B} L={cfg.L} V={cfg.V} K={cfg.K} "
                                f"n_max={cfg.n_max} layers={cfg.layers} Hq={cfg.Hq} Hkv={cfg.Hkv} "
                                f"D={cfg.D} ctx={cfg.ctx} page={cfg.page}",
-                   "global_batch": cfg.B, "seq_len": int(ctx_h.max()), "parallelism": "replicas",
+                   "global_batch": cfg.B, "seq_len": int(rs.ctx_h.max()),
+                   "parallelism": "replicas",
                    "l2": f"inputs larger than L2: {cfg.layers} distinct KV layers, "
-                         f"{kv_bytes / 1e9:.1f} GB per step",
+                         f"{rs.kv_bytes / 1e9:.1f} GB per step",
                    "n_nodes": int(sel_h["n_nodes"][0]),
                    "mode": args.mode,
                    "select_plus_one_layer_round_us": round(one_layer_us, 2),
@@ -570,12 +713,24 @@ def run_ours(args):
         "gpu_launches": launches,
         "clocks": clk,
     }
+    if sweep is not None:
+        line["sweep"] = sweep
     if rank == 0 and not args.no_cpu_baseline:
         cb = run_cpu_baseline(args, steps=1, warmup=0, sample_layers=args.sample_layers)
         line["cpu_baseline"] = {"value": round(1.0 / cb["scaled_s"][0], 4), "unit": "rounds/s",
                                 "cores": 1, "kind": "oracle",
                                 "sample": sample_desc(cfg, args.sample_layers)
                                 + f"; wall {cb['wall_s'][0]:.1f} s"}
+        cores = os.cpu_count() or 1
+        if cores > 1:
+            cb = run_cpu_baseline(args, steps=1, warmup=0, sample_layers=args.sample_layers,
+                                  cores=cores)
+            line["cpu_baseline_all_cores"] = {
+                "value": round(1.0 / cb["scaled_s"][0], 4), "unit": "rounds/s", "cores": cores,
+                "kind": "oracle",
+                "sample": sample_desc(cfg, args.sample_layers)
+                + f"; stage 5 spread over {cores} processes by (request, head); "
+                  f"wall {cb['wall_s'][0]:.1f} s"}
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:
@@ -643,7 +798,7 @@ def run_reference(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="qwen3_8b")
@@ -654,6 +809,9 @@ def main():
                     choices=["taps", "no_scorer", "budget_fill", "ddtree"],
                     help="selection preset: TAPS, or one of its ablations")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-sweep", action="store_true",
+                    help="skip the other configurations (budget sweep, Qwen3-4B, batch 32, long)")
+    ap.add_argument("--cpu-cores", type=int, default=1, help=argparse.SUPPRESS)
     ap.add_argument("--only-topk", action="store_true",
                     help="time stage 1 alone on the workload's logits (profiling aid)")
     ap.add_argument("--no-cpu-baseline", action="store_true")

@@ -122,6 +122,9 @@ int taps_topk_marginals(const void* logits, int dtype, int64_t row_stride,
  * its kernel runs. Every call shares the one array per device, so calls that
  * overlap on the GPU (different streams, or different host threads without
  * ordering) race: serialise them.
+ * The library caches per-device state for the life of the process (this
+ * array's address, kernel attributes, cluster capacities), so resetting a
+ * device (cudaDeviceReset) between calls into the library is not supported.
  * Limits: B * L <= TAPS_NOALLOC_MAX_ROWS (4096); beyond it the call returns
  * TAPS_ERR_UNSUPPORTED and launches nothing. Other limits as above.
  * ---------------------------------------------------------------------- */
@@ -135,7 +138,8 @@ int taps_topk_marginals_noalloc(const void* logits, int dtype, int64_t row_strid
 /* ------------------------------------------------------------------------
  * taps_score_reach - Sec. 4.2, Eq. 1 and Algorithm 1: for every parent of
  * the candidate trie, q_cond(parent -> child) = softmax over the K siblings
- * of the scorer logit of each edge.
+ * of the scorer logit of each edge; optionally Eq. 2, the reach
+ * q_reach = product of q_cond along the path, of a caller-given node list.
  *
  * The candidate trie: every node at depth d has the same K children, the
  * top-K tokens of position d; the root (depth 0) carries root_tok[b].
@@ -159,7 +163,19 @@ int taps_topk_marginals_noalloc(const void* logits, int dtype, int64_t row_strid
  *                        device f32 buffer: tok_emb[vocab][E], dep_emb[max_depth][E],
  *                        W1[H][3E+2], b1[H], w2[H], w_lp[1], packed in that
  *                        order. Token ids must be < vocab; max_depth > L.
- * Limits: K <= 32, L <= 31, E <= 32, H <= 64.
+ *
+ * Reach of an explicit node list (Eq. 2), optional: paths, path_len and
+ * path_reach are all NULL with M == 0, or all given with M >= 1.
+ *   paths      [B, M, L] uint8: node m of request b is the trie node reached
+ *              from the root by top-K slots paths[b, m, 0 .. path_len[b, m]).
+ *   path_len   [B, M] int32, its depth (0 = the root).
+ *   path_reach [B, M] f32, out: product of q_cond along the path, one IEEE
+ *              round-to-nearest multiply per edge, root to leaf: bit-identical
+ *              to the reach taps_select_subtree computes for the same node.
+ *              A length outside [0, L], or a slot >= K among the first
+ *              path_len entries, names no node of the trie: reach 0.
+ *   It runs after q_cond is complete, in a second kernel on the same stream.
+ * Limits: K <= 32, L <= 31, E <= 32, H <= 64, B * M < 2^31 - 256.
  * ---------------------------------------------------------------------- */
 typedef struct taps_scorer_params {
   int kind;
@@ -172,7 +188,9 @@ typedef struct taps_scorer_params {
 
 int taps_score_reach(const int32_t* root_tok, const int32_t* topk_ids, const float* topk_logp,
                      const float* entropy, int B, int L, int K,
-                     const taps_scorer_params* params, float* q_cond, void* stream);
+                     const taps_scorer_params* params, float* q_cond,
+                     const uint8_t* paths, const int32_t* path_len, int M,
+                     float* path_reach, void* stream);
 
 /* ------------------------------------------------------------------------
  * taps_select_subtree - Eq. 2 (reach = product of q_cond along the path),

@@ -59,7 +59,8 @@ lib.taps_topk_marginals_workspace_bytes.argtypes = [_I, _I, _I, _I]
 lib.taps_topk_marginals_workspace_bytes.restype = _SZ
 lib.taps_topk_marginals.argtypes = [_P, _I, _I64, _I, _I, _I, _I, _P, _P, _P, _P, _P, _SZ, _P]
 lib.taps_topk_marginals.restype = _I
-lib.taps_score_reach.argtypes = [_P, _P, _P, _P, _I, _I, _I, ctypes.POINTER(ScorerParams), _P, _P]
+lib.taps_score_reach.argtypes = [_P, _P, _P, _P, _I, _I, _I, ctypes.POINTER(ScorerParams), _P,
+                                 _P, _P, _I, _P, _P]
 lib.taps_score_reach.restype = _I
 lib.taps_select_subtree.argtypes = [_P, _P, _P, _P, _I, _I, _I, ctypes.POINTER(SelectParams),
                                     _P, _P, _P, _P, _P, _P, _P, _P, _P]
@@ -173,20 +174,31 @@ def scorer_params(kind: str, weights: torch.Tensor | None = None, emb_dim=0, hid
 
 
 def taps_score_reach(root_tok, topk_ids, topk_logp, entropy, params: ScorerParams, out=None,
-                     stream=None):
-    """Stage 2: q_cond [B, L, K, K] f32."""
+                     paths=None, path_len=None, path_reach=None, stream=None):
+    """Stage 2: q_cond [B, L, K, K] f32. With ``paths`` [B, M, L] uint8 slots and
+    ``path_len`` [B, M] int32, also the reach of those nodes (Eq. 2), returned as
+    (q_cond, path_reach [B, M] f32)."""
     B, L, K = topk_ids.shape
     _need(root_tok, torch.int32, (B,), "root_tok")
     _need(topk_ids, torch.int32, (B, L, K), "topk_ids")
     _need(topk_logp, torch.float32, (B, L, K), "topk_logp")
     _need(entropy, torch.float32, (B, L), "entropy")
-    q = out if out is not None else torch.empty((B, L, K, K), dtype=torch.float32,
-                                                 device=topk_ids.device)
+    dev = topk_ids.device
+    q = out if out is not None else torch.empty((B, L, K, K), dtype=torch.float32, device=dev)
+    M = 0
+    if paths is not None:
+        M = paths.shape[1] if paths.dim() == 3 else -1
+        _need(paths, torch.uint8, (B, M, L), "paths")
+        _need(path_len, torch.int32, (B, M), "path_len")
+        if path_reach is None:
+            path_reach = torch.empty((B, M), dtype=torch.float32, device=dev)
+        _need(path_reach, torch.float32, (B, M), "path_reach")
     st = lib.taps_score_reach(_ptr(root_tok), _ptr(topk_ids), _ptr(topk_logp), _ptr(entropy),
-                              B, L, K, ctypes.byref(params), _ptr(q),
-                              _stream(stream, topk_ids.device))
+                              B, L, K, ctypes.byref(params), _ptr(q), _ptr(paths),
+                              _ptr(path_len), M, _ptr(path_reach) if paths is not None else None,
+                              _stream(stream, dev))
     _check("taps_score_reach", st)
-    return q
+    return (q, path_reach) if paths is not None else q
 
 
 def taps_select_subtree(q_cond, topk_ids, root_tok, ctx_len, lambda1, lambda2, tau, n_max,

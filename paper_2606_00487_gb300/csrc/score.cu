@@ -128,6 +128,45 @@ score_kernel(const int32_t* __restrict__ root_tok, const int32_t* __restrict__ i
   }
 }
 
+// Eq. 2 for an explicit list of nodes: reach = product of q_cond along the
+// path, one IEEE f32 multiply per edge, root to leaf (the operations and order
+// of the selection's reach). One thread per (request, path); the slots are
+// known up front, so the path's q_cond loads are independent of each other.
+__global__ void __launch_bounds__(256)
+path_reach_kernel(const float* __restrict__ q_cond, const uint8_t* __restrict__ paths,
+                  const int32_t* __restrict__ path_len, int B, int L, int K, int M,
+                  float* __restrict__ path_reach) {
+  dep_enter();
+  const int64_t e = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (e >= static_cast<int64_t>(B) * M) return;
+  const int b = static_cast<int>(e / M);
+  const int n = path_len[e];
+  float r = 0.f;   // not a node of the trie
+  if (n >= 0 && n <= L) {
+    const uint8_t* p = paths + e * L;
+    const float* qb = q_cond + static_cast<int64_t>(b) * L * K * K;
+    float qv[TAPS_MAX_L];
+    bool ok = true;
+    int prev = 0;   // depth-1 children hang off the root, row 0
+#pragma unroll
+    for (int d = 0; d < TAPS_MAX_L; ++d) {
+      if (d < n) {
+        const int j = p[d];
+        ok = ok && j < K;
+        qv[d] = j < K ? qb[(d * K + prev) * K + j] : 0.f;
+        prev = j < K ? j : 0;
+      }
+    }
+    if (ok) {
+      r = 1.0f;
+#pragma unroll
+      for (int d = 0; d < TAPS_MAX_L; ++d)
+        if (d < n) r = __fmul_rn(r, qv[d]);
+    }
+  }
+  path_reach[e] = r;
+}
+
 }  // namespace
 }  // namespace taps
 
@@ -135,9 +174,17 @@ using namespace taps;
 
 extern "C" int taps_score_reach(const int32_t* root_tok, const int32_t* topk_ids,
                                 const float* topk_logp, const float* entropy, int B, int L, int K,
-                                const taps_scorer_params* params, float* q_cond, void* stream) {
+                                const taps_scorer_params* params, float* q_cond,
+                                const uint8_t* paths, const int32_t* path_len, int M,
+                                float* path_reach, void* stream) {
   if (!root_tok || !topk_ids || !topk_logp || !q_cond || !params) return TAPS_ERR_INVALID_ARG;
   if (B <= 0 || L <= 0 || K <= 0) return TAPS_ERR_INVALID_ARG;
+  // the path list is all or nothing
+  const bool want_paths = paths || path_len || path_reach;
+  if (want_paths && (!paths || !path_len || !path_reach || M <= 0)) return TAPS_ERR_INVALID_ARG;
+  if (!want_paths && M != 0) return TAPS_ERR_INVALID_ARG;
+  if (want_paths && static_cast<int64_t>(B) * M > (static_cast<int64_t>(1) << 31) - 256)
+    return TAPS_ERR_UNSUPPORTED;
   if (K > TAPS_MAX_K || L > TAPS_MAX_L || B > 65535) return TAPS_ERR_UNSUPPORTED;
   int kind = params->kind;
   int E = 0, H = 0;
@@ -159,5 +206,12 @@ extern "C" int taps_score_reach(const int32_t* root_tok, const int32_t* topk_ids
                  params->max_depth, static_cast<const float*>(params->weights), q_cond) !=
       cudaSuccess)
     return TAPS_ERR_CUDA;
+  if (want_paths) {
+    const int64_t n = static_cast<int64_t>(B) * M;
+    if (launch_dep(path_reach_kernel, dim3(static_cast<unsigned>((n + 255) / 256)), dim3(256), 0,
+                   static_cast<cudaStream_t>(stream), q_cond, paths, path_len, B, L, K, M,
+                   path_reach) != cudaSuccess)
+      return TAPS_ERR_CUDA;
+  }
   return launch_status();
 }

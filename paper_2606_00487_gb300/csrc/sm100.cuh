@@ -305,6 +305,13 @@ __device__ __forceinline__ void tma_store_4d(const CUtensorMap* map, uint32_t sr
       "r"(x), "r"(y), "r"(z), "r"(w), "r"(src_smem)
       : "memory");
 }
+// 1D bulk copy shared -> global of `bytes` (multiple of 16, both addresses
+// 16-byte aligned), tracked by the bulk-group mechanism.
+__device__ __forceinline__ void bulk_store(void* dst, uint32_t src_smem, uint32_t bytes) {
+  asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(dst),
+               "r"(src_smem), "r"(bytes)
+               : "memory");
+}
 __device__ __forceinline__ void bulk_commit() {
   asm volatile("cp.async.bulk.commit_group;" ::: "memory");
 }

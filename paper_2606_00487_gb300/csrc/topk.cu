@@ -13,6 +13,7 @@
 // reset after use) merges the partials by rank and writes the row's outputs.
 // No CTA waits on another.
 #include <algorithm>
+#include <atomic>
 #include <mutex>
 
 #include "common.cuh"
@@ -592,13 +593,17 @@ void launch(const void* logits, int64_t row_stride, const Plan& p, int V, int K,
   uint64_t* keys = p.chunks > 1 ? reinterpret_cast<uint64_t*>(ws + w.keys) : nullptr;
   unsigned* tk = p.chunks > 1 ? reinterpret_cast<unsigned*>(ws + w.tickets) : nullptr;
   // the copy ring exceeds the default 48 KB of dynamic shared memory: raise
-  // the limit once per device (setting it twice from racing threads is harmless)
-  static bool ring_attr[64] = {};
+  // the limit once per device. The flags are atomics because the entry points
+  // may be called from several host threads; two threads setting the same
+  // attribute at once is harmless.
+  static std::atomic<bool> ring_attr[64];
   int dev = 0;
-  if (cudaGetDevice(&dev) == cudaSuccess && dev >= 0 && dev < 64 && !ring_attr[dev]) {
-    cudaFuncSetAttribute(topk_marginals_kernel<KP, T>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                         static_cast<int>(kRingBytes));
-    ring_attr[dev] = true;
+  if (cudaGetDevice(&dev) == cudaSuccess && dev >= 0 && dev < 64 &&
+      !ring_attr[dev].load(std::memory_order_acquire)) {
+    if (cudaFuncSetAttribute(topk_marginals_kernel<KP, T>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(kRingBytes)) == cudaSuccess)
+      ring_attr[dev].store(true, std::memory_order_release);
   }
   launch_dep(topk_marginals_kernel<KP, T>, grid, dim3(kThreads), vec_ok ? kRingBytes : 0, s,
              static_cast<const T*>(logits), row_stride, V, K, p.chunks, vec_ok, ids, logp, lse,

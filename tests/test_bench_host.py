@@ -61,3 +61,42 @@ def test_mode_presets_and_metric_names():
         assert cfg.layers == (W.CONFIGS[name].layers if layers is None else layers)
     assert "Qwen3-8B" in bench.metric_name("qwen3_8b")
     assert "LLaMA-3.1-8B" in bench.metric_name("llama31_8b")
+
+
+def test_all_cores_oracle_split_covers_every_row_once():
+    """The all-cores CPU baseline splits stage 5 by (request, head) over worker
+    processes; the workers' outputs, summed, equal the serial oracle's."""
+    cfg = W.CONFIGS["tiny"].with_(B=2)
+    bench._attn_worker_init(cfg)
+    inp = bench._W["inp"]
+    rng = np.random.default_rng(8)
+    n_nodes = np.array([16, 7], np.int32)
+    parent = np.full((2, 16), -1, np.int32)
+    for b in range(2):
+        for i in range(1, n_nodes[b]):
+            parent[b, i] = rng.integers(0, i)
+    mask = O.build_tree_mask(parent, n_nodes, 16)
+    ref, _ = O.tree_verify_attn(inp["q"], inp["k"], inp["v"], inp["bt"], inp["ctx"], n_nodes, mask)
+    pairs = [(b, h) for b in range(cfg.B) for h in range(cfg.Hq)]
+    n_w = 3
+    parts = [bench._attn_worker_rows((pairs[i::n_w], n_nodes, mask)) for i in range(n_w)]
+    assert np.array_equal(sum(parts), ref)
+    bench._W.clear()
+
+
+def test_roofline_names_the_binding_bound():
+    """N = 64 at the Qwen3-8B shape is HBM-bound (its byte floor is the higher
+    one), N = 256 tensor-bound (4 flops per byte per node: intensity ~ 4 n)."""
+    peaks = (6704.5, 1911.0, 1736.0, "measured")
+    for n, bound in ((64, "hbm"), (256, "tensor")):
+        cfg = W.CONFIGS["qwen3_8b"].with_(n_max=n)
+        rs = bench.RoundSetup.__new__(bench.RoundSetup)
+        rs.cfg = cfg
+        rs.ctx_h = np.array([4096])
+        depth = np.full((1, n), 4, np.int64)
+        depth[0, 0] = 0
+        rs.sel_h = {"n_nodes": np.array([n]), "depth": depth}
+        rl = rs.roofline(36 * 0.010, peaks)          # 10 us per layer
+        assert rl["bound"] == bound
+        assert rl["avg_launch_us"] == 10.0
+        assert abs(rl["hbm_frac"] - rl["algorithmic_bytes_per_launch"] / 10e-6 / 1e9 / 6704.5) < 1e-4

@@ -79,15 +79,27 @@ def test_topk_rejects_bad_arguments(lib):
 
 def test_score_select_mask_accept_reject_bad_arguments(lib):
     tb = _b()
+    score = tb.lib.taps_score_reach
+    nopath = (None, None, 0, None)
     sp = tb.ScorerParams(tb.TAPS_SCORER_MLP, 16, 32, 100, 3, None)
-    assert tb.lib.taps_score_reach(FAKE, FAKE, FAKE, FAKE, 1, 2, 4, ctypes.byref(sp), FAKE,
-                                   None) == 1                       # no weights
+    assert score(FAKE, FAKE, FAKE, FAKE, 1, 2, 4, ctypes.byref(sp), FAKE, *nopath,
+                 None) == 1                                          # no weights
     sp = tb.ScorerParams(tb.TAPS_SCORER_MLP, 64, 32, 100, 3, FAKE)
-    assert tb.lib.taps_score_reach(FAKE, FAKE, FAKE, FAKE, 1, 2, 4, ctypes.byref(sp), FAKE,
-                                   None) == 2                       # E > 32
+    assert score(FAKE, FAKE, FAKE, FAKE, 1, 2, 4, ctypes.byref(sp), FAKE, *nopath,
+                 None) == 2                                          # E > 32
     sp = tb.ScorerParams(tb.TAPS_SCORER_MLP, 16, 32, 100, 2, FAKE)
-    assert tb.lib.taps_score_reach(FAKE, FAKE, FAKE, FAKE, 1, 2, 4, ctypes.byref(sp), FAKE,
-                                   None) == 1                       # max_depth <= L
+    assert score(FAKE, FAKE, FAKE, FAKE, 1, 2, 4, ctypes.byref(sp), FAKE, *nopath,
+                 None) == 1                                          # max_depth <= L
+    # the path list (Eq. 2 reach of given nodes) is all or nothing
+    sp = tb.ScorerParams(tb.TAPS_SCORER_MARGINAL, 0, 0, 0, 0, None)
+    assert score(FAKE, FAKE, FAKE, FAKE, 1, 2, 4, ctypes.byref(sp), FAKE, FAKE, None, 3,
+                 FAKE, None) == 1                                    # path_len missing
+    assert score(FAKE, FAKE, FAKE, FAKE, 1, 2, 4, ctypes.byref(sp), FAKE, FAKE, FAKE, 0,
+                 FAKE, None) == 1                                    # M = 0 with paths
+    assert score(FAKE, FAKE, FAKE, FAKE, 1, 2, 4, ctypes.byref(sp), FAKE, None, None, 5,
+                 None, None) == 1                                    # M without paths
+    assert score(FAKE, FAKE, FAKE, FAKE, 2, 2, 4, ctypes.byref(sp), FAKE, FAKE, FAKE,
+                 2 ** 30, FAKE, None) == 2                           # B * M too large
     sel = tb.lib.taps_select_subtree
     args = [FAKE] * 8
     for (l1, l2, tau, n), code in (((0.0, 0.1, 0.0, 8), 1), ((1.0, -0.1, 0.0, 8), 1),

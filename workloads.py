@@ -103,10 +103,21 @@ _S_LOGITS, _S_SCORER, _S_CTX, _S_ROOT, _S_TARGET, _S_KV, _S_Q, _S_PAGES = range(
 
 
 def round_to_bf16(x: np.ndarray) -> np.ndarray:
-    """Round float32 values to the nearest bfloat16 (ties to even); returns float32."""
-    bits = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32).astype(np.uint64)
-    rounded = ((bits + 0x7FFF + ((bits >> 16) & 1)) >> 16) << 16
-    return rounded.astype(np.uint32).view(np.float32)
+    """Round float32 values to the nearest bfloat16 (ties to even); returns float32.
+
+    Works on the uint32 bit patterns in place: adding 0x7FFF plus the lowest
+    kept bit cannot overflow 32 bits for any non-NaN value (the inputs here
+    never hold NaN)."""
+    bits = np.array(x, dtype=np.float32, copy=True).view(np.uint32)
+    flat = bits.reshape(-1)
+    step = 1 << 22
+    for a in range(0, flat.size, step):
+        c = flat[a:a + step]
+        lsb = (c >> 16) & 1
+        c += np.uint32(0x7FFF)
+        c += lsb
+        c &= np.uint32(0xFFFF0000)
+    return bits.view(np.float32)
 
 
 def bf16_bits(x: np.ndarray) -> np.ndarray:
