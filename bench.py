@@ -585,12 +585,18 @@ def run_ours(args):
                                                       r.lambda2, r.tau, r.n_max, out=r.sel),
         "s4_mask": lambda: taps.taps_build_tree_mask(r.sel["parent"], r.sel["n_nodes"],
                                                      out=r.mask),
+        "s2_s3_s4_fused": lambda: taps.taps_score_select_mask(
+            root, r.ids, r.logp, r.entropy, ctx, r.scorer, r.lambda1, r.lambda2, r.tau, r.n_max,
+            out=(r.q_cond, r.sel, r.mask)),
         "s5_attention_one_layer": lambda: r.verify_layer(q0, k0, v0, b0, ctx, outs[0]),
         "s6_accept": lambda: r.accept(target),
     }
     # the latency-bound stages back to back in one graph (what a round spends
-    # outside top-K and verification)
+    # outside top-K and verification): as the round runs them (scoring,
+    # selection and mask in one launch, then acceptance), and one launch per stage
     stage_fns["s2_s3_s4_s6_in_one_graph"] = lambda: [stage_fns[k]() for k in (
+        "s2_s3_s4_fused", "s6_accept")]
+    stage_fns["s2_s3_s4_s6_one_launch_per_stage"] = lambda: [stage_fns[k]() for k in (
         "s2_score", "s3_select", "s4_mask", "s6_accept")]
     stage_us = {}
     for name, fn in stage_fns.items():

@@ -14,6 +14,8 @@
  *   taps_accept            Sec. 4.1 and Limitations (greedy, temperature 0,
  *                          lossless acceptance of the longest matching path)
  *
+ * taps_score_select_mask runs the second to fourth steps in two launches.
+ *
  * and two steps that follow verification in the decoding loop:
  *
  *   taps_target_greedy_accept  Limitations (temperature 0: the target's
@@ -224,6 +226,26 @@ int taps_select_subtree(const float* q_cond, const int32_t* topk_ids, const int3
                         int32_t* n_nodes, int32_t* parent, int32_t* depth, int32_t* token,
                         int32_t* slot, int32_t* pos_id, float* reach, float* utility,
                         void* stream);
+
+/* ------------------------------------------------------------------------
+ * taps_score_select_mask - stages 2-4 of a round (Sec. 4.2, Eq. 1-3,
+ * Algorithm 1, Sec. 4.3) in two launches: exactly the outputs of
+ * taps_score_reach (q_cond, no path list), then taps_select_subtree, then
+ * taps_build_tree_mask, with the same arguments, limits and errors, bit for
+ * bit. The scorer keeps its own launch (one CTA per position and request,
+ * which spreads a batch-1 round over many SMs); the selection and the mask
+ * share one CTA per request, which builds the mask from the tree in shared
+ * memory.
+ * q_cond [B, L, K, K], the selection outputs [B] / [B, n_max] and mask
+ * [B, n_max, ceil(n_max / 32)] are written as the separate calls write them.
+ * ---------------------------------------------------------------------- */
+int taps_score_select_mask(const int32_t* root_tok, const int32_t* topk_ids,
+                           const float* topk_logp, const float* entropy, const int32_t* ctx_len,
+                           int B, int L, int K, const taps_scorer_params* scorer,
+                           const taps_select_params* select, float* q_cond, int32_t* n_nodes,
+                           int32_t* parent, int32_t* depth, int32_t* token, int32_t* slot,
+                           int32_t* pos_id, float* reach, float* utility, uint32_t* mask,
+                           void* stream);
 
 /* ------------------------------------------------------------------------
  * taps_build_tree_mask - the ancestor-or-self relation that tree attention

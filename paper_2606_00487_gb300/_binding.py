@@ -226,6 +226,47 @@ def taps_select_subtree(q_cond, topk_ids, root_tok, ctx_len, lambda1, lambda2, t
     return out
 
 
+lib.taps_score_select_mask.argtypes = [_P, _P, _P, _P, _P, _I, _I, _I,
+                                       ctypes.POINTER(ScorerParams), ctypes.POINTER(SelectParams),
+                                       _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P]
+lib.taps_score_select_mask.restype = _I
+
+
+def taps_score_select_mask(root_tok, topk_ids, topk_logp, entropy, ctx_len, params: ScorerParams,
+                           lambda1, lambda2, tau, n_max, out=None, stream=None):
+    """Stages 2-4 (scoring, then selection and mask in one launch): returns (q_cond [B, L, K, K],
+    selection dict as taps_select_subtree, mask [B, n_max, ceil(n_max/32)]).
+    ``out`` = (q_cond, sel, mask) preallocated, or None."""
+    B, L, K = topk_ids.shape
+    _need(root_tok, torch.int32, (B,), "root_tok")
+    _need(topk_ids, torch.int32, (B, L, K), "topk_ids")
+    _need(topk_logp, torch.float32, (B, L, K), "topk_logp")
+    _need(entropy, torch.float32, (B, L), "entropy")
+    _need(ctx_len, torch.int32, (B,), "ctx_len")
+    dev = topk_ids.device
+    W = (n_max + 31) // 32
+    if out is None:
+        sel = {"n_nodes": torch.empty(B, dtype=torch.int32, device=dev)}
+        for k in ("parent", "depth", "token", "slot", "pos_id"):
+            sel[k] = torch.empty((B, n_max), dtype=torch.int32, device=dev)
+        for k in ("reach", "utility"):
+            sel[k] = torch.empty((B, n_max), dtype=torch.float32, device=dev)
+        out = (torch.empty((B, L, K, K), dtype=torch.float32, device=dev), sel,
+               torch.empty((B, n_max, W), dtype=torch.int32, device=dev))
+    q, sel, mask = out
+    _need(q, torch.float32, (B, L, K, K), "q_cond")
+    _need(mask, torch.int32, (B, n_max, W), "mask")
+    p = SelectParams(float(lambda1), float(lambda2), float(tau), int(n_max))
+    st = lib.taps_score_select_mask(_ptr(root_tok), _ptr(topk_ids), _ptr(topk_logp),
+                                    _ptr(entropy), _ptr(ctx_len), B, L, K, ctypes.byref(params),
+                                    ctypes.byref(p), _ptr(q), _ptr(sel["n_nodes"]),
+                                    _ptr(sel["parent"]), _ptr(sel["depth"]), _ptr(sel["token"]),
+                                    _ptr(sel["slot"]), _ptr(sel["pos_id"]), _ptr(sel["reach"]),
+                                    _ptr(sel["utility"]), _ptr(mask), _stream(stream, dev))
+    _check("taps_score_select_mask", st)
+    return q, sel, mask
+
+
 def taps_build_tree_mask(parent, n_nodes, out=None, stream=None):
     """Stage 4: mask [B, n_max, ceil(n_max/32)] uint32 (returned as int32 storage)."""
     B, n_max = parent.shape

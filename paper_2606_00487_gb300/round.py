@@ -2,7 +2,9 @@
 
 Sequencing only: the six stages run in the order of Sec. 4.1 (top-K
 marginals -> scoring -> selection -> mask -> per-layer tree verification ->
-acceptance), each as one call into libtaps.so on the caller's stream. With
+acceptance) as calls into libtaps.so on the caller's stream; scoring,
+selection and the mask are one call (taps_score_select_mask, whose selection
+and mask share one launch). With
 the target's verify logits at hand, acceptance can instead take the greedy
 token of every node from them (accept_greedy), and commit_kv moves the
 accepted path's K/V into place for the next round. All
@@ -76,11 +78,20 @@ class TapsRound:
             self.scorer_weights = scorer_weights
             self.scorer = tb.scorer_params("mlp", scorer_weights, emb_dim, hidden, V,
                                            max_depth if max_depth is not None else L + 1)
-        self.launches_per_select = 4
+        self.launches_per_select = 3
         self.launches_per_layer = 1 + (1 if tb.lib.taps_tree_verify_attn_workspace_bytes(
             B, n_max, Hq, Hkv, D, max_ctx) > 0 else 0)
 
     def select(self, logits, root_tok, ctx_len, stream=None):
+        """Stage 1, scoring, then selection and mask in one launch."""
+        tb.taps_topk_marginals(logits, self.K, out=(self.ids, self.logp, self.lse, self.entropy),
+                               ws=self.ws_topk, stream=stream)
+        tb.taps_score_select_mask(root_tok, self.ids, self.logp, self.entropy, ctx_len,
+                                  self.scorer, self.lambda1, self.lambda2, self.tau, self.n_max,
+                                  out=(self.q_cond, self.sel, self.mask), stream=stream)
+
+    def select_staged(self, logits, root_tok, ctx_len, stream=None):
+        """The same results with one launch per stage (stages 1-4)."""
         tb.taps_topk_marginals(logits, self.K, out=(self.ids, self.logp, self.lse, self.entropy),
                                ws=self.ws_topk, stream=stream)
         tb.taps_score_reach(root_tok, self.ids, self.logp, self.entropy, self.scorer,

@@ -110,6 +110,26 @@ def test_score_select_mask_accept_reject_bad_arguments(lib):
     p = tb.SelectParams(1.0, 0.1, 0.0, 8)
     assert sel(FAKE, FAKE, FAKE, FAKE, 1, 32, 4, ctypes.byref(p), *args, None) == 2   # L > 31
     assert tb.lib.taps_build_tree_mask(FAKE, FAKE, 1, 600, FAKE, None) == 2
+    # stages 2-4 in one launch: the same checks as the separate calls
+    fused = tb.lib.taps_score_select_mask
+    outs = [FAKE] * 10
+    sp = tb.ScorerParams(tb.TAPS_SCORER_MARGINAL, 0, 0, 0, 0, None)
+    for (l1, l2, tau, n), code in (((0.0, 0.1, 0.0, 8), 1), ((1.0, -0.1, 0.0, 8), 1),
+                                   ((1.0, 0.1, 0.0, 0), 1), ((1.0, 0.1, 0.0, 513), 2)):
+        p = tb.SelectParams(l1, l2, tau, n)
+        assert fused(FAKE, FAKE, FAKE, FAKE, FAKE, 1, 4, 4, ctypes.byref(sp), ctypes.byref(p),
+                     *outs, None) == code
+    p = tb.SelectParams(1.0, 0.1, 0.0, 8)
+    assert fused(FAKE, FAKE, FAKE, FAKE, FAKE, 1, 32, 4, ctypes.byref(sp), ctypes.byref(p),
+                 *outs, None) == 2                                    # L > 31
+    sp = tb.ScorerParams(tb.TAPS_SCORER_MLP, 16, 32, 100, 3, None)
+    assert fused(FAKE, FAKE, FAKE, FAKE, FAKE, 1, 2, 4, ctypes.byref(sp), ctypes.byref(p),
+                 *outs, None) == 1                                    # no weights
+    sp = tb.ScorerParams(7, 0, 0, 0, 0, None)
+    assert fused(FAKE, FAKE, FAKE, FAKE, FAKE, 1, 2, 4, ctypes.byref(sp), ctypes.byref(p),
+                 *outs, None) == 1                                    # unknown scorer
+    assert fused(FAKE, FAKE, FAKE, FAKE, None, 1, 2, 4, ctypes.byref(sp), ctypes.byref(p),
+                 *outs, None) == 1                                    # no ctx_len
     assert tb.lib.taps_build_tree_mask(None, FAKE, 1, 8, FAKE, None) == 1
     assert tb.lib.taps_accept(FAKE, FAKE, FAKE, FAKE, 1, 8, 40, FAKE, FAKE, FAKE, None) == 2
     assert tb.lib.taps_accept(FAKE, FAKE, None, FAKE, 1, 8, 4, FAKE, FAKE, FAKE, None) == 1

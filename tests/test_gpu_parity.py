@@ -327,6 +327,76 @@ def test_select_underflowing_reach(taps):
 
 
 # ---------------------------------------------------------------------------
+# Stages 2-4 through taps_score_select_mask (selection and mask in one launch)
+# ---------------------------------------------------------------------------
+
+def _scorer(taps, kind, cfg):
+    if kind != "mlp":
+        return taps.scorer_params(kind), None
+    w = W.make_scorer_weights(cfg)
+    return taps.scorer_params("mlp", dt(w["packed"]), w["E"], w["H"], w["V"], w["max_depth"]), w
+
+
+def _check_fused(taps, ids, logp, ent, root, ctx, sp, l1, l2, tau, n_max):
+    """The fused launch equals the three separate calls bit for bit, and its
+    selection and mask equal the oracle's on its own q_cond."""
+    args = (dt(root), dt(ids), dt(logp), dt(ent))
+    q1 = taps.taps_score_reach(*args, sp)
+    s1 = taps.taps_select_subtree(q1, dt(ids), dt(root), dt(ctx), l1, l2, tau, n_max)
+    m1 = taps.taps_build_tree_mask(s1["parent"], s1["n_nodes"])
+    q2, s2, m2 = taps.taps_score_select_mask(dt(root), dt(ids), dt(logp), dt(ent), dt(ctx), sp,
+                                              l1, l2, tau, n_max)
+    torch.cuda.synchronize()
+    assert torch.equal(q1.view(torch.int32), q2.view(torch.int32))
+    for k in SEL_KEYS:
+        assert torch.equal(s1[k], s2[k]), k
+    assert torch.equal(m1, m2)
+    ref = O.select_subtree(host(q2), ids, root, ctx, l1, l2, tau, n_max)
+    for k in SEL_KEYS:
+        np.testing.assert_array_equal(host(s2[k]), ref[k], err_msg=k)
+    np.testing.assert_array_equal(host(m2).view(np.uint32),
+                                  O.build_tree_mask(ref["parent"], ref["n_nodes"], n_max))
+    return q2, ref
+
+
+@pytest.mark.parametrize("name,n_max,kind,tau", [("tiny", 16, "mlp", 0.0),
+                                                 ("qwen3_8b", 64, "mlp", 0.0),
+                                                 ("qwen3_8b", 256, "mlp", 0.0),
+                                                 ("qwen3_8b", 256, "mlp", 2e-2),
+                                                 ("qwen3_4b", 512, "marginal", 0.0),
+                                                 ("qwen3_8b", 64, "marginal_product", 0.0),
+                                                 ("long", 256, "mlp", 0.0),
+                                                 ("llama31_8b", 64, "mlp", 0.0),
+                                                 ("batched", 64, "mlp", 0.0)])
+def test_fused_score_select_mask(taps, name, n_max, kind, tau):
+    cfg = W.CONFIGS[name]
+    x, ids, logp, ent, root = _stage1_inputs(cfg, B=cfg.B if name == "batched" else min(cfg.B, 2))
+    sp, w = _scorer(taps, kind, cfg)
+    ctx = W.make_ctx_lens(cfg, B=x.shape[0])
+    l2 = 0.0 if kind == "marginal_product" else cfg.lambda2
+    q, ref = _check_fused(taps, ids, logp, ent, root, ctx, sp, cfg.lambda1, l2, tau, n_max)
+    np.testing.assert_allclose(host(q), O.score_qcond(root, ids, logp, ent, kind, w),
+                               rtol=1e-5, atol=1e-7)
+    if tau > 0:
+        assert (ref["n_nodes"] < n_max).any()
+
+
+def test_fused_large_shape(taps):
+    """The largest tables the limits allow in practice: L = 24, K = 32,
+    n_max = 512 (ranking passes over 512 + appended entries)."""
+    rng = np.random.default_rng(23)
+    B, L, K = 2, 24, 32
+    ids = np.stack([np.stack([rng.permutation(100000)[:K] for _ in range(L)])
+                    for _ in range(B)]).astype(np.int32)
+    logp = -np.sort(rng.exponential(3.0, size=(B, L, K)), axis=-1).astype(np.float32)
+    ent = rng.random((B, L)).astype(np.float32) * 5
+    root = rng.integers(0, 100000, size=B).astype(np.int32)
+    ctx = np.array([10, 2000], np.int32)
+    _check_fused(taps, ids, logp, ent, root, ctx, taps.scorer_params("marginal"), 1.0, 0.05,
+                 0.0, 512)
+
+
+# ---------------------------------------------------------------------------
 # Stage 4
 # ---------------------------------------------------------------------------
 
