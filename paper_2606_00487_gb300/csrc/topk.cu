@@ -168,6 +168,60 @@ __device__ void warp_top(const uint64_t* cand, int n, uint64_t* out, int lane) {
   }
 }
 
+// Candidate c of cand[0, n) goes to out[rank] when its rank (keys above it,
+// equal keys ordered by index; only empty entries, 0, can be equal) is below
+// KP. One thread per candidate; the loads are broadcasts.
+template <int KP>
+__device__ __forceinline__ void rank_into(const uint64_t* cand, int n, int c, uint64_t* out) {
+  const uint64_t mine = cand[c];
+  int rank = 0;
+  int i = 0;
+  for (; i + 3 < n; i += 4) {
+    const uint64_t a0 = cand[i], a1 = cand[i + 1], a2 = cand[i + 2], a3 = cand[i + 3];
+    rank += (a0 > mine || (a0 == mine && i < c)) + (a1 > mine || (a1 == mine && i + 1 < c)) +
+            (a2 > mine || (a2 == mine && i + 2 < c)) + (a3 > mine || (a3 == mine && i + 3 < c));
+  }
+  for (; i < n; ++i) rank += cand[i] > mine || (cand[i] == mine && i < c);
+  if (rank < KP) out[rank] = mine;
+}
+
+// Top-KP of cand[0, n) into out[0, KP), descending, called by every thread
+// of the CTA. thr is a key that at least KP of the candidates reach (0 when
+// none is known): a candidate below it has KP candidates above it, so only
+// the few at or above it are compacted into comp (one shared atomic per warp)
+// and ranked among themselves. *ncomp is 0 on entry and is left at 0. When
+// more than cap candidates reach thr, they are ranked with warp maxima.
+template <int KP>
+__device__ void select_top(const uint64_t* cand, int n, uint64_t thr, uint64_t* comp, int cap,
+                           int* ncomp, uint64_t* out, uint64_t* part) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  for (int i0 = warp * 32; i0 < n; i0 += kThreads) {
+    const int i = i0 + lane;
+    const uint64_t k = i < n ? cand[i] : 0ull;
+    const bool keep = i < n && k >= thr;
+    const unsigned b = __ballot_sync(kFullMask, keep);
+    int base = 0;
+    if (lane == 0 && b) base = atomicAdd(ncomp, __popc(b));
+    base = __shfl_sync(kFullMask, base, 0);
+    const int idx = base + __popc(b & ((1u << lane) - 1u));
+    if (keep && idx < cap) comp[idx] = k;
+  }
+  __syncthreads();
+  const int m = *ncomp;
+  if (m <= cap) {
+    for (int c = tid; c < m; c += kThreads) rank_into<KP>(comp, m, c, out);
+  } else {
+    // each warp reduces a slice of at most 256 keys, then warp 0 the results
+    const int slice = (n + kWarps - 1) / kWarps;
+    const int lo = min(n, warp * slice), hi = min(n, lo + slice);
+    warp_top<KP>(cand + lo, hi - lo, part + warp * KP, lane);
+    __syncthreads();
+    if (warp == 0) warp_top<KP>(part, kWarps * KP, out, lane);
+  }
+  __syncthreads();
+  if (tid == 0) *ncomp = 0;
+}
+
 __device__ __forceinline__ Stats warp_stats(Stats s) {
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) {
@@ -216,7 +270,12 @@ topk_marginals_kernel(const T* __restrict__ logits, int64_t row_stride, int V, i
   // row are >= it, so a key below it can be in no top-K (keys are unique, and
   // the key itself sits in the list of the warp that holds it)
   __shared__ unsigned long long s_thr;
-  if (threadIdx.x == 0) s_thr = 0ull;
+  __shared__ int s_ncomp;          // entries in s_part compacted by select_top
+  __shared__ unsigned long long s_rthr;
+  if (threadIdx.x == 0) {
+    s_thr = 0ull;
+    s_ncomp = 0;
+  }
   __syncthreads();
 
   const int row = blockIdx.y;
@@ -446,8 +505,28 @@ topk_marginals_kernel(const T* __restrict__ logits, int64_t row_stride, int V, i
       // threshold's (a lower value has a lower key whatever its token id)
       const uint64_t shared_thr = *reinterpret_cast<volatile unsigned long long*>(&s_thr);
       const uint64_t thr = shared_thr > kth ? shared_thr : kth;
-      const float thr_v = thr ? ordered_to_f32(static_cast<uint32_t>(thr >> 32)) : -INFINITY;
+      float thr_v = thr ? ordered_to_f32(static_cast<uint32_t>(thr >> 32)) : -INFINITY;
       if (__any_sync(kFullMask, (live[0] || live[1]) && (thr == 0 || tmax >= thr_v))) {
+        // Warm-up (this warp's list not yet full, no CTA threshold): the
+        // KP-th largest lane maximum of the tile, counted with multiplicity,
+        // is a value that at least KP of the tile's elements reach, so no
+        // element below it can be in the tile's top-KP (nor in the top-KP of
+        // the tile and the list). Found by 32-bit warp maxima over the lanes.
+        int warm_left = 0;
+        if (thr == 0) {
+          uint32_t cur = (live[0] || live[1]) ? f32_to_ordered(tmax) : 0u;
+          uint32_t t = 0u;
+          int need = KP;
+          while (need > 0) {
+            const uint32_t m = __reduce_max_sync(kFullMask, cur);
+            if (m == 0u) break;                    // fewer than KP live lanes
+            need -= __popc(__ballot_sync(kFullMask, cur == m));
+            t = m;
+            if (cur == m) cur = 0u;
+          }
+          if (need <= 0) thr_v = ordered_to_f32(t);
+          warm_left = need;
+        }
         // elements whose value reaches the threshold's value: only they can
         // hold a key above it
         uint32_t flag = 0;
@@ -455,7 +534,8 @@ topk_marginals_kernel(const T* __restrict__ logits, int64_t row_stride, int V, i
         for (int i = 0; i < EPT; ++i)
           flag |= (live[i / VE] && vals[i] >= thr_v) ? (1u << i) : 0u;
         const int nflag = __popc(flag);
-        if (thr != 0 && __reduce_add_sync(kFullMask, static_cast<unsigned>(nflag)) <= kFewKeys) {
+        const unsigned few = thr != 0 ? kFewKeys : (warm_left <= 0 ? KP + kFewKeys : 0);
+        if (__reduce_add_sync(kFullMask, static_cast<unsigned>(nflag)) <= few) {
           // few: visit only the element slots some lane flagged, build those
           // keys, and insert the ones above the threshold
 #pragma unroll
@@ -534,10 +614,11 @@ topk_marginals_kernel(const T* __restrict__ logits, int64_t row_stride, int V, i
   st = warp_stats(st);
   if (lane == 0) s_wstats[warp] = st;
   __syncthreads();
+  // the CTA's top-KP: only the warp candidates at or above the CTA threshold
+  // (the largest K-th key any warp holds) can be in it
+  select_top<KP>(s_cand, kWarps * KP, s_thr, s_part, kWarps * 32, &s_ncomp, s_top, s_part);
 
   if (warp == 0) {
-    warp_top<KP>(s_cand, kWarps * KP, s_top, lane);
-    __syncwarp();
     Stats cs = s_wstats[0];
     for (int w = 1; w < kWarps; ++w) cs = stats_merge(cs, s_wstats[w]);
     if (chunks == 1) {
@@ -558,26 +639,29 @@ topk_marginals_kernel(const T* __restrict__ logits, int64_t row_stride, int V, i
   __syncthreads();
   if (!s_last) return;
 
-  // ---- last CTA of this row: merge every chunk's partial record
+  // ---- last CTA of this row: merge every chunk's partial record. The
+  // partial statistics are loaded with the keys, in one round trip.
   __threadfence();
   const int64_t rec0 = static_cast<int64_t>(row) * chunks;
-  for (int i = tid; i < chunks * KP; i += kThreads) s_cand[i] = __ldcg(ws_keys + rec0 * KP + i);
-  __syncthreads();
-  {
-    // each warp reduces a slice of at most 256 keys, then warp 0 the 8 results
-    const int n = chunks * KP, slice = (n + kWarps - 1) / kWarps;
-    const int lo = min(n, warp * slice), hi = min(n, lo + slice);
-    warp_top<KP>(s_cand + lo, hi - lo, s_part + warp * KP, lane);
-  }
-  __syncthreads();
-  if (warp == 0) warp_top<KP>(s_part, kWarps * KP, s_top, lane);
-  __syncthreads();
+  const int n = chunks * KP;
+  for (int i = tid; i < n; i += kThreads) s_cand[i] = __ldcg(ws_keys + rec0 * KP + i);
+  Stats cs{-INFINITY, 0.f, 0.f};
   if (warp == 0) {
-    Stats cs{-INFINITY, 0.f, 0.f};
+    // every chunk's list is sorted: the largest of their K-th keys is a key
+    // that at least KP candidates reach
+    uint64_t kmax = 0ull;
     for (int c = lane; c < chunks; c += 32) {
       float4 p = __ldcg(ws_stats + rec0 + c);
       cs = stats_merge(cs, Stats{p.x, p.y, p.z});
+      const uint64_t kk = __ldcg(ws_keys + (rec0 + c) * KP + KP - 1);
+      kmax = kk > kmax ? kk : kmax;
     }
+    kmax = warp_max_u64(kmax);
+    if (lane == 0) s_rthr = kmax;
+  }
+  __syncthreads();
+  select_top<KP>(s_cand, n, s_rthr, s_part, kWarps * 32, &s_ncomp, s_top, s_part);
+  if (warp == 0) {
     cs = warp_stats(cs);
     write_row<KP>(row, K, s_top, cs, lane, ids, logp, lse, ent);
     if (lane == 0) tickets[row] = 0u;
