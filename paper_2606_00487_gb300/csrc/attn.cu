@@ -483,7 +483,6 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
     };
     int pgn = page_id(0);
     for (int j = 0; j < n_tiles; ++j) {
-      if (__any_sync(kFullMask, *abort_flag != 0)) { ok = false; break; }
       // visible columns of this row in tile j: on a valid page, inside the
       // chunk, and for tree nodes on the row's ancestor path
       const uint32_t live = __ballot_sync(kFullMask, pgn >= 0 && pgn < a.num_pages);
@@ -509,11 +508,17 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
           }
         }
       }
+      // S of tile j. A shared-memory access waits behind the tensor core's
+      // operand reads, so the abort flag is read only when S is not ready
+      // at the first test (every wait is bounded in any case).
       const int u = j % kSBufs;
-      if (!__all_sync(kFullMask, mbar_wait(&s_full[u], (j / kSBufs) & 1))) {
-        if (lane == 0) set_fault(abort_flag, a.status, TAPS_DEVFAULT_TIMEOUT);
-        ok = false;
-        break;
+      if (!__all_sync(kFullMask, mbar_try_wait(&s_full[u], (j / kSBufs) & 1))) {
+        if (__any_sync(kFullMask, *abort_flag != 0)) { ok = false; break; }
+        if (!__all_sync(kFullMask, mbar_wait(&s_full[u], (j / kSBufs) & 1))) {
+          if (lane == 0) set_fault(abort_flag, a.status, TAPS_DEVFAULT_TIMEOUT);
+          ok = false;
+          break;
+        }
       }
       tc_fence_after();
       uint32_t sv[128];

@@ -1,6 +1,7 @@
 // Internal helpers shared by the TAPS CUDA sources (not part of the C ABI).
 #pragma once
 
+#include <atomic>
 #include <cuda_runtime.h>
 #include <cuda_bf16.h>
 #include <stdint.h>
@@ -43,6 +44,25 @@ inline cudaError_t launch_dep(void (*kernel)(KArgs...), dim3 grid, dim3 block, s
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
+// Raise the dynamic shared-memory limit of a kernel once per device (atomic
+// flags: calls may come from several host threads).
+template <typename Kern>
+bool smem_limit(Kern kernel, size_t bytes, std::atomic<int>* done) {
+  if (bytes <= 48 * 1024) return true;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return false;
+  // the flag holds the largest size set so far (+1)
+  if (done[dev].load(std::memory_order_acquire) > static_cast<int>(bytes)) return true;
+  if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           static_cast<int>(bytes)) != cudaSuccess)
+    return false;
+  int prev = done[dev].load(std::memory_order_relaxed);
+  while (prev <= static_cast<int>(bytes) &&
+         !done[dev].compare_exchange_weak(prev, static_cast<int>(bytes) + 1)) {
+  }
+  return true;
 }
 
 inline int launch_status() {

@@ -14,6 +14,7 @@ namespace taps {
 namespace {
 
 constexpr int kThreads = 256;
+constexpr int kWarps = kThreads / 32;
 
 __global__ void __launch_bounds__(kThreads)
 score_kernel(const int32_t* __restrict__ root_tok, const int32_t* __restrict__ ids,
@@ -38,93 +39,135 @@ score_kernel(const int32_t* __restrict__ root_tok, const int32_t* __restrict__ i
   float* s_D = s_C + K * H;                  // [H]    per-position pre-activation
   int* s_ptok = reinterpret_cast<int*>(s_D + H);  // [K]
   int* s_ctok = s_ptok + K;                       // [K]
+  // MLP operands staged in shared memory (first layer rows padded to an odd
+  // stride, so that the threads of a warp, one hidden unit each, read
+  // different banks)
+  const int FP = F | 1;
+  float* s_W1 = reinterpret_cast<float*>(s_ctok + K);   // [H][FP]
+  float* s_b1 = s_W1 + H * FP;                          // [H]
+  float* s_w2 = s_b1 + H;                               // [H + 1]
+  float* s_dep = s_w2 + H + 1;                          // [E] depth embedding of d + 1
+  float* s_emb = s_dep + E;                             // [np + K][E] parents', then children's
 
+  const bool mlp = kind == TAPS_SCORER_MLP;
+  const float* tok_emb = w;
+  const float* dep_emb = tok_emb + static_cast<int64_t>(vocab) * E;
+  const float* W1 = dep_emb + static_cast<int64_t>(max_depth) * E;
+  const float* b1 = W1 + H * F;
+  const float* w2 = b1 + H;
   for (int j = tid; j < K; j += kThreads) {
     s_logp[j] = logp[row0 + j];
     s_ctok[j] = ids[row0 + j];
     s_ptok[j] = d == 0 ? root_tok[b] : ids[row0 - K + j];
   }
+  if (mlp) {
+    for (int i = tid; i < H * F; i += kThreads) s_W1[(i / F) * FP + i % F] = W1[i];
+    for (int i = tid; i < 2 * H + 1; i += kThreads) s_b1[i] = b1[i];   // b1, then w2 and its logp weight
+    const float* drow = dep_emb + static_cast<int64_t>(min(d + 1, max_depth - 1)) * E;
+    for (int i = tid; i < E; i += kThreads) s_dep[i] = drow[i];
+  }
   __syncthreads();
 
-  if (kind != TAPS_SCORER_MLP) {
+  if (!mlp) {
     for (int e = tid; e < np * K; e += kThreads) s_ell[e] = s_logp[e % K];
   } else {
-    const float* tok_emb = w;
-    const float* dep_emb = tok_emb + static_cast<int64_t>(vocab) * E;
-    const float* W1 = dep_emb + static_cast<int64_t>(max_depth) * E;
-    const float* b1 = W1 + H * F;
-    const float* w2 = b1 + H;
-    const float w_lp = w2[H];
+    const float w_lp = s_w2[H];
     const float ent = entropy[static_cast<int64_t>(b) * L + d];
+    // the token embedding rows of the parents and the children (0 for an id
+    // outside the vocabulary, whose dot product is then skipped)
+    for (int i = tid; i < (np + K) * E; i += kThreads) {
+      const int rrow = i / E, e = i % E;
+      const int tok = rrow < np ? s_ptok[rrow] : s_ctok[rrow - np];
+      s_emb[i] = (tok >= 0 && tok < vocab) ? tok_emb[static_cast<int64_t>(tok) * E + e] : 0.f;
+    }
+    __syncthreads();
     // per-parent, per-child and per-position parts of W1 f + b1
     const int items = (np + K) * H + H;
     for (int it = tid; it < items; it += kThreads) {
-      const float* wrow;
-      const float* emb;
       float acc;
-      int tok;
       if (it < np * H) {                       // parent part
-        int i = it / H, h = it % H;
-        tok = s_ptok[i];
-        wrow = W1 + h * F;
-        emb = (tok >= 0 && tok < vocab) ? tok_emb + static_cast<int64_t>(tok) * E : nullptr;
+        const int i = it / H, h = it % H;
+        const int tok = s_ptok[i];
+        const float* wrow = s_W1 + h * FP;
+        const float* emb = s_emb + i * E;
         acc = 0.f;
-        if (emb)
+        if (tok >= 0 && tok < vocab)
           for (int e = 0; e < E; ++e) acc = fmaf(wrow[e], emb[e], acc);
         s_P[i * H + h] = acc;
       } else if (it < (np + K) * H) {          // child part (+ logp column)
-        int r = it - np * H;
-        int j = r / H, h = r % H;
-        tok = s_ctok[j];
-        wrow = W1 + h * F + E;
-        emb = (tok >= 0 && tok < vocab) ? tok_emb + static_cast<int64_t>(tok) * E : nullptr;
+        const int r = it - np * H;
+        const int j = r / H, h = r % H;
+        const int tok = s_ctok[j];
+        const float* wrow = s_W1 + h * FP + E;
+        const float* emb = s_emb + (np + j) * E;
         acc = 0.f;
-        if (emb)
+        if (tok >= 0 && tok < vocab)
           for (int e = 0; e < E; ++e) acc = fmaf(wrow[e], emb[e], acc);
-        acc = fmaf(W1[h * F + 3 * E], s_logp[j], acc);
+        acc = fmaf(s_W1[h * FP + 3 * E], s_logp[j], acc);
         s_C[j * H + h] = acc;
       } else {                                 // per-position part
-        int h = it - (np + K) * H;
-        wrow = W1 + h * F + 2 * E;
-        emb = dep_emb + static_cast<int64_t>(min(d + 1, max_depth - 1)) * E;
-        acc = b1[h];
-        for (int e = 0; e < E; ++e) acc = fmaf(wrow[e], emb[e], acc);
-        acc = fmaf(W1[h * F + 3 * E + 1], ent, acc);
+        const int h = it - (np + K) * H;
+        const float* wrow = s_W1 + h * FP + 2 * E;
+        acc = s_b1[h];
+        for (int e = 0; e < E; ++e) acc = fmaf(wrow[e], s_dep[e], acc);
+        acc = fmaf(s_W1[h * FP + 3 * E + 1], ent, acc);
         s_D[h] = acc;
       }
     }
     __syncthreads();
-    // edge logits: one warp reduction over the hidden units per edge
-    const int nw = kThreads / 32;
-    for (int e = warp; e < np * K; e += nw) {
-      int i = e / K, j = e % K;
-      float acc = 0.f;
-      for (int h = lane; h < H; h += 32) {
-        float a = s_P[i * H + h] + s_C[j * H + h] + s_D[h];
-        acc = fmaf(w2[h], fmaxf(a, 0.f), acc);
+    // edge logits: one warp reduction over the hidden units per edge, four
+    // edges of a warp at a time so that their reductions overlap
+    for (int e0 = warp; e0 < np * K; e0 += 4 * kWarps) {
+      float acc[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int e = e0 + u * kWarps;
+        acc[u] = 0.f;
+        if (e < np * K) {
+          const int i = e / K, j = e % K;
+          for (int h = lane; h < H; h += 32) {
+            const float a = s_P[i * H + h] + s_C[j * H + h] + s_D[h];
+            acc[u] = fmaf(s_w2[h], fmaxf(a, 0.f), acc[u]);
+          }
+        }
       }
 #pragma unroll
-      for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(kFullMask, acc, off);
-      if (lane == 0) s_ell[e] = fmaf(w_lp, s_logp[j], acc);
+      for (int off = 16; off > 0; off >>= 1)
+#pragma unroll
+        for (int u = 0; u < 4; ++u) acc[u] += __shfl_xor_sync(kFullMask, acc[u], off);
+      if (lane == 0)
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int e = e0 + u * kWarps;
+          if (e < np * K) s_ell[e] = fmaf(w_lp, s_logp[e % K], acc[u]);
+        }
     }
   }
   __syncthreads();
 
-  // sibling-wise softmax, one thread per parent row (the marginal-product
-  // kind takes each child's marginal probability as it is)
+  // sibling-wise softmax, one warp per parent row and one lane per child
+  // (K <= 32); the marginal-product kind takes each child's marginal
+  // probability as it is
   float* out = q_cond + (static_cast<int64_t>(b) * L + d) * K * K;
-  for (int i = tid; i < K; i += kThreads) {
-    if (i < np && kind == TAPS_SCORER_MARGINAL_PRODUCT) {
-      for (int j = 0; j < K; ++j) out[i * K + j] = expf(s_ell[i * K + j]);
-    } else if (i < np) {
-      float m = -INFINITY;
-      for (int j = 0; j < K; ++j) m = fmaxf(m, s_ell[i * K + j]);
-      float sum = 0.f;
-      for (int j = 0; j < K; ++j) sum += expf(s_ell[i * K + j] - m);
-      for (int j = 0; j < K; ++j) out[i * K + j] = __fdiv_rn(expf(s_ell[i * K + j] - m), sum);
-    } else {
-      for (int j = 0; j < K; ++j) out[i * K + j] = 0.f;
+  const bool in = lane < K;
+  for (int i = warp; i < K; i += kWarps) {
+    if (i >= np) {
+      if (in) out[i * K + lane] = 0.f;
+      continue;
     }
+    const float x = in ? s_ell[i * K + lane] : -INFINITY;
+    if (kind == TAPS_SCORER_MARGINAL_PRODUCT) {
+      if (in) out[i * K + lane] = expf(x);
+      continue;
+    }
+    float m = x;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) m = fmaxf(m, __shfl_xor_sync(kFullMask, m, off));
+    const float ex = in ? expf(x - m) : 0.f;
+    float sum = ex;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(kFullMask, sum, off);
+    if (in) out[i * K + lane] = __fdiv_rn(ex, sum);
   }
 }
 
@@ -167,6 +210,8 @@ path_reach_kernel(const float* __restrict__ q_cond, const uint8_t* __restrict__ 
   path_reach[e] = r;
 }
 
+std::atomic<int> g_score_smem[64];
+
 }  // namespace
 }  // namespace taps
 
@@ -198,8 +243,15 @@ extern "C" int taps_score_reach(const int32_t* root_tok, const int32_t* topk_ids
   } else if (kind != TAPS_SCORER_MARGINAL && kind != TAPS_SCORER_MARGINAL_PRODUCT) {
     return TAPS_ERR_INVALID_ARG;
   }
+  // q/logits, logp, per-parent/child/position parts, token ids, then (MLP) the
+  // staged first layer (rows padded to an odd stride), b1, w2, the depth
+  // embedding and the parents' and children's token embeddings
   size_t smem = sizeof(float) * (K * K + K + 2 * K * std::max(H, 1) + std::max(H, 1)) +
                 sizeof(int) * 2 * K;
+  if (kind == TAPS_SCORER_MLP)
+    smem += sizeof(float) * (static_cast<size_t>(H) * ((3 * E + 2) | 1) + 2 * H + 1 + E +
+                             static_cast<size_t>(2 * K) * E);
+  if (!smem_limit(score_kernel, smem, g_score_smem)) return TAPS_ERR_CUDA;
   dim3 grid(L, B);
   if (launch_dep(score_kernel, grid, dim3(kThreads), smem, static_cast<cudaStream_t>(stream),
                  root_tok, topk_ids, topk_logp, entropy, L, K, kind, E, H, params->vocab,

@@ -444,25 +444,6 @@ select_mask_kernel(const float* __restrict__ q_cond, const int* __restrict__ ids
   }
 }
 
-// Raise the dynamic shared-memory limit of a kernel once per device (atomic
-// flags: calls may come from several host threads).
-template <typename Kern>
-bool smem_limit(Kern kernel, size_t bytes, std::atomic<int>* done) {
-  if (bytes <= 48 * 1024) return true;
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return false;
-  // the flag holds the largest size set so far (+1)
-  if (done[dev].load(std::memory_order_acquire) > static_cast<int>(bytes)) return true;
-  if (cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           static_cast<int>(bytes)) != cudaSuccess)
-    return false;
-  int prev = done[dev].load(std::memory_order_relaxed);
-  while (prev <= static_cast<int>(bytes) &&
-         !done[dev].compare_exchange_weak(prev, static_cast<int>(bytes) + 1)) {
-  }
-  return true;
-}
-
 std::atomic<int> g_select_smem[64];
 std::atomic<int> g_select_mask_smem[64];
 
