@@ -5,7 +5,9 @@ of Sec. 4.1 on the GPU: top-K marginals, scoring, selection, mask, tree
 verification attention for every layer of the target, acceptance. The round
 is captured as three CUDA graphs (stages 1-4, the per-layer attention calls,
 stage 6) and replayed; CUDA events between the graphs time the attention
-stage live for the roofline figure.
+stage live for the roofline figure. The end-to-end figure (``e2e``) replays the
+whole round with its uploads from pinned host memory and the read of its
+results as one graph per round, waiting for the results before the next round.
 
 Workload (default): Qwen3-8B shape, batch 1, draft block L=16, vocab 151936,
 bf16 drafter logits (Zipf s=1.1 with position temperature 0.6 -> 1.4), top-K 8,
@@ -36,6 +38,9 @@ sys.path.insert(0, ROOT)
 FALLBACK_HBM_GBS = 6800.0
 FALLBACK_BF16_TFLOPS = 1900.0
 FALLBACK_BF16_TFLOPS_SUSTAINED = 1700.0
+# the end-to-end round uploads the tree queries in this many groups of layers,
+# each group of verification layers waiting only for its own
+E2E_QUERY_GROUPS = 4
 
 
 def attn_source_sha256():
@@ -439,6 +444,37 @@ class RoundSetup:
         torch.cuda.synchronize()
         self.stream = torch.cuda.current_stream(dev)
 
+    def capture_e2e(self, res_pin, groups):
+        """One round with its host copies as one CUDA graph: the head upload,
+        the queries in ``groups`` groups of layers on a copy stream (each group
+        of verification layers waits only for its own queries), the round, and
+        the read of its results into ``res_pin``."""
+        import torch
+        r, inp, cfg, s = self.r, self.inp, self.cfg, self.s
+        cs = torch.cuda.Stream(device=s.device)
+        per = (cfg.layers + groups - 1) // groups
+        spans = [(k * per, min(cfg.layers, (k + 1) * per)) for k in range(groups)
+                 if k * per < cfg.layers]
+        evs = [torch.cuda.Event() for _ in spans]
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=s):
+            cs.wait_stream(s)
+            inp.upload_head(s)
+            for (a, b), e in zip(spans, evs):
+                inp.upload_queries(cs, a, b)
+                e.record(cs)
+            r.select(self.logits, self.root, self.ctx, s)
+            for (a, b), e in zip(spans, evs):
+                s.wait_event(e)
+                for li in range(a, b):
+                    q, kc, vc, b_t = self.layers[li]
+                    r.verify_layer(q, kc, vc, b_t, self.ctx, self.outs[li], s)
+            r.accept(self.target, s)
+            s.wait_stream(cs)
+            r.download(res_pin, s)
+        torch.cuda.synchronize()
+        return g
+
     def step(self, ev_a=None, ev_b=None):
         self.g_pre.replay()
         if ev_a is not None:
@@ -625,30 +661,23 @@ def run_ours(args):
     e2e = None
     inp = rs.inp
     if not args.no_e2e:
-        # the host staging buffer holds every input of a round (logits, root
-        # tokens, the 36 layers' tree queries, target tokens): one upload per
-        # round, then the round, then one read of its results
-        # The head (logits, root and target tokens) goes first on the compute
-        # stream; the queries of all layers travel on a copy stream while the
-        # selection stages run, and verification waits for them.
+        # The host staging buffer holds every input of a round (logits, root
+        # tokens, the 36 layers' tree queries, target tokens). Each round, as
+        # one CUDA graph: the head (logits, root and target tokens) uploads on
+        # the compute stream; the queries upload on a copy stream in
+        # E2E_QUERY_GROUPS groups of layers while the selection stages run, and
+        # each group of verification layers waits only for its own queries;
+        # then acceptance and one read of the round's results. The host waits
+        # for that read before the next round starts, as a decoding loop must.
         torch.cuda.synchronize()
         inp.host_buf.copy_(inp.device_buf)
         res_pin = torch.empty(r.results.shape, dtype=r.results.dtype, pin_memory=True)
         h2d = inp.nbytes
         d2h = res_pin.numel() * res_pin.element_size()
-        copy_stream = torch.cuda.Stream(device=dev)
-        q_ready = torch.cuda.Event()
+        g_e2e = rs.capture_e2e(res_pin, E2E_QUERY_GROUPS)
 
         def e2e_step():
-            copy_stream.wait_stream(stream)        # the previous round is done with the queries
-            inp.upload_head(stream)
-            inp.upload_queries(copy_stream)
-            q_ready.record(copy_stream)
-            rs.g_pre.replay()
-            stream.wait_event(q_ready)
-            rs.g_attn.replay()
-            rs.g_post.replay()
-            r.download(res_pin, stream)
+            g_e2e.replay()
             stream.synchronize()
 
         for _ in range(args.warmup):
