@@ -192,7 +192,6 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
 
   // ---- set-up that reads no input: may overlap the previous grid's tail
   const Plan& pl = a.plan;
-  const int b = blockIdx.z;
   const int kv = blockIdx.y / pl.m_blocks;
   const int mb = blockIdx.y % pl.m_blocks;
   const int split = blockIdx.x;
@@ -234,6 +233,22 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
   }
   __syncthreads();   // barriers initialised
   pdl_wait();
+
+  // Requests longest first: blocks start in launch order, the request index
+  // (z) slowest, so with 2 to 32 requests block row z takes the request of
+  // z-th largest length (ctx_len + n_nodes, ties by index) and the long ones
+  // do not end up in the last wave. Every warp ranks the lengths itself.
+  int b = blockIdx.z;
+  if (gridDim.z > 1 && gridDim.z <= 32) {
+    const int B = static_cast<int>(gridDim.z);
+    const int len = lane < B ? a.ctx_len[lane] + min(max(a.n_nodes[lane], 0), a.n_max) : -1;
+    int rank = 0;
+    for (int j = 0; j < B; ++j) {
+      const int lj = __shfl_sync(kFullMask, len, j);
+      rank += (lj > len || (lj == len && j < lane)) ? 1 : 0;
+    }
+    b = __ffs(__ballot_sync(kFullMask, lane < B && rank == static_cast<int>(blockIdx.z))) - 1;
+  }
 
   // ---- inputs. The request's lengths and the chunk's page ids are
   // requested together; then Q and each producer's first tile leave at once,
