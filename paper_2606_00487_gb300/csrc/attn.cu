@@ -13,14 +13,14 @@
 // ever leaves the chip and no second kernel is needed.
 //
 // Inside a CTA (8 warps):
-//   warps 0, 2  TMA producers (one thread each): warp 0 loads Q once (4D box)
-//            and the K tiles into a 3-stage ring, warp 2 the V tiles into a
-//            2-stage ring, one contiguous bulk copy per 16-token page of a
-//            128-token tile; the chunk's page ids are first copied to shared
-//            memory by the whole of warp 0. The cache uses the TAPS page
-//            layout (see taps_pack_kv_pages): a (page, head) block is stored
-//            exactly as the tensor core reads it, 8-token groups of 128-byte
-//            swizzled rows, so one copy per page feeds the MMAs directly.
+//   warps 0, 2  producers: warp 0 streams the K tiles, warp 2 the V tiles,
+//            each into a 2-stage ring, one bulk copy per 16-token page of a
+//            128-token tile (lane p copies page p). The cache uses the TAPS
+//            page layout (see taps_pack_kv_pages): a (page, head) block is
+//            stored exactly as the tensor core reads it, 8-token groups of
+//            128-byte swizzled rows, so one copy per page feeds the MMAs.
+//   warp 3   copies the chunk's page ids to shared memory, then loads Q (4D
+//            tensor-map boxes).
 //   warp 1   allocates all 512 TMEM columns and issues every tcgen05.mma.
 //            S = Q K^T (M=128, N=128, K=D) goes to one of three S buffers;
 //            O += P V (M=128, N=D, K=16 per page) reads P from TMEM. After
@@ -36,6 +36,8 @@
 //            reduction writes it.
 // TMEM columns: O at [0, D), S (fp32) and then P (bf16 pairs) of buffer u at
 // [128 + 128 u, 256 + 128 u), u = 0, 1, 2; tile j uses buffer j mod 3.
+// With 2 to 32 requests in a launch, block rows take the requests longest
+// first, so that long requests do not start in the last wave.
 // Every wait is bounded; a wait that runs out sets TAPS_DEVFAULT_TIMEOUT and
 // the CTA winds down (waiting for its own copies and MMAs) before freeing TMEM.
 // Launches use programmatic dependent launch: a grid may start its set-up
