@@ -507,13 +507,47 @@ def _sampled_check(q, kc, vc, bt, ctx, nn, mask, out, rng, per_req=6):
 
 def test_attention_parity_many_tiles(taps):
     """Every output row against the oracle where each CTA streams several
-    128-token tiles (ctx 4000, 64 nodes: chunks of 4-5 tiles, a ragged last
-    page), so the S/P buffers, the K and V rings and the lazy rescale all
-    wrap around."""
+    128-token tiles (ctx 4000, 64 nodes: chunks of 4-6 tiles, a ragged last
+    page), so the S/P buffers and the K and V rings wrap around (the lazy
+    rescale has its own test below)."""
     cfg = W.CONFIGS["qwen3_8b"]
     ctx_a = np.array([4000], np.int32)
     nn = np.array([64], np.int32)
     q, kc, vc, bt, mask = _attn_inputs(cfg, 1, nn, ctx_a, 64)
+    out, lse = _run_attn(taps, q, kc, vc, bt, ctx_a, nn, mask)
+    ref, ref_lse = O.tree_verify_attn(_f32(q), _f32(kc), _f32(vc), bt, ctx_a, nn, mask)
+    assert np.abs(_f32(out) - ref).max() <= ATTN_ATOL
+    np.testing.assert_allclose(host(lse)[0, :64], ref_lse[0, :64], rtol=1e-4, atol=1e-4)
+
+
+def test_attention_lazy_rescale(taps):
+    """Keys of every third 128-token tile scaled by 4, so that within a chunk
+    a row's running maximum jumps by more than 8 (base 2) from one tile to the
+    next and the output accumulator is rescaled in TMEM (the lazy-rescale
+    path, which unscaled synthetic keys never reach); every row against the
+    oracle."""
+    cfg = W.CONFIGS["qwen3_8b"]
+    ctx_a = np.array([4000], np.int32)
+    nn = np.array([64], np.int32)
+    rng = np.random.default_rng(0)
+    parent = _tree(rng, 64, 64)
+    mask = O.build_tree_mask(parent, nn, 64)
+    bt, num_pages = W.make_block_table(cfg, ctx_a, 64)
+    kn, vn = W.make_kv_numpy(cfg, num_pages)
+    pos = np.arange(int(ctx_a[0]))
+    spike = (pos // 128) % 3 == 2
+    kn = kn.copy()
+    kn[bt[0][pos[spike] // 16], :, pos[spike] % 16, :] *= 4
+    q, kc, vc = bf(W.make_q_numpy(cfg, 1, 64)), bf(kn), bf(vn)
+    # the premise: a spike tile's maximum exceeds the tile before it by more
+    # than 8 (base 2) in most rows of KV head 0
+    group = cfg.Hq // cfg.Hkv
+    rows = _f32(q)[0, :, :group, :].reshape(-1, cfg.D)
+    k0 = _f32(kc)[bt[0][pos // 16], 0, pos % 16, :]
+    s2 = rows @ k0.T * (np.log2(np.e) / np.sqrt(cfg.D))
+    tmax = np.stack([s2[:, t:t + 128].max(axis=1) for t in range(0, 3840, 128)], axis=1)
+    jumps = tmax[:, 2::3] > tmax[:, 1::3][:, :tmax[:, 2::3].shape[1]] + 8
+    assert jumps.any(axis=1).mean() > 0.5
     out, lse = _run_attn(taps, q, kc, vc, bt, ctx_a, nn, mask)
     ref, ref_lse = O.tree_verify_attn(_f32(q), _f32(kc), _f32(vc), bt, ctx_a, nn, mask)
     assert np.abs(_f32(out) - ref).max() <= ATTN_ATOL
