@@ -445,33 +445,13 @@ class RoundSetup:
         self.stream = torch.cuda.current_stream(dev)
 
     def capture_e2e(self, res_pin, groups):
-        """One round with its host copies as one CUDA graph: the head upload,
-        the queries in ``groups`` groups of layers on a copy stream (each group
-        of verification layers waits only for its own queries), the round, and
-        the read of its results into ``res_pin``."""
+        """One round with its host copies as one CUDA graph, through
+        TapsRound.capture_round_graph: the head upload, the queries in
+        ``groups`` groups of layers on a copy stream, the round, and the read
+        of its results into ``res_pin``."""
         import torch
-        r, inp, cfg, s = self.r, self.inp, self.cfg, self.s
-        cs = torch.cuda.Stream(device=s.device)
-        per = (cfg.layers + groups - 1) // groups
-        spans = [(k * per, min(cfg.layers, (k + 1) * per)) for k in range(groups)
-                 if k * per < cfg.layers]
-        evs = [torch.cuda.Event() for _ in spans]
-        g = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(g, stream=s):
-            cs.wait_stream(s)
-            inp.upload_head(s)
-            for (a, b), e in zip(spans, evs):
-                inp.upload_queries(cs, a, b)
-                e.record(cs)
-            r.select(self.logits, self.root, self.ctx, s)
-            for (a, b), e in zip(spans, evs):
-                s.wait_event(e)
-                for li in range(a, b):
-                    q, kc, vc, b_t = self.layers[li]
-                    r.verify_layer(q, kc, vc, b_t, self.ctx, self.outs[li], s)
-            r.accept(self.target, s)
-            s.wait_stream(cs)
-            r.download(res_pin, s)
+        g = self.r.capture_round_graph(self.inp, self.ctx, self.layers, self.outs, res_pin,
+                                       groups, stream=self.s)
         torch.cuda.synchronize()
         return g
 

@@ -142,6 +142,57 @@ class TapsRound:
             self.verify_layer(q, kc, vc, bt, ctx_len, o, stream)
         self.accept(target_tok, stream)
 
+    def capture_round_graph(self, inputs, ctx_len, layers, outs, host_results, groups=4,
+                            stream=None):
+        """Capture one whole round with its host copies as one CUDA graph and
+        return it; each ``replay()`` then runs a round from what the host
+        buffer of ``inputs`` (a RoundInputs) holds at that moment.
+
+        In the graph: the head (logits, root and target tokens) uploads on the
+        capture stream; the queries upload on a second stream in ``groups``
+        groups of layers while stages 1-4 run, and each group of verification
+        layers waits only for its own queries; then acceptance and one
+        device-to-host copy of ``results`` into ``host_results`` (pinned,
+        results.numel() int32). ``layers`` is a list of (q, k_cache, v_cache,
+        block_table) whose q must be the device views ``inputs.dev["q"][i]``,
+        so that the graph's uploads feed them; ``outs`` holds one output per
+        layer. ``stream`` is the capture stream (a fresh one by default; it
+        must not be the legacy default stream). The caller synchronizes the
+        stream it replays on before reading ``host_results``."""
+        if len(layers) != inputs.layers or len(outs) != inputs.layers:
+            raise ValueError("one (q, k_cache, v_cache, block_table) and one output per layer")
+        for li, (q, _, _, _) in enumerate(layers):
+            if q.data_ptr() != inputs.dev["q"][li].data_ptr():
+                raise ValueError(f"layer {li}: q is not the upload buffer's view of that layer")
+        if host_results.numel() != self.results.numel() or not host_results.is_pinned():
+            raise ValueError("host_results must be pinned with results.numel() elements")
+        groups = max(1, min(int(groups), inputs.layers))
+        per = (inputs.layers + groups - 1) // groups
+        spans = [(a, min(inputs.layers, a + per)) for a in range(0, inputs.layers, per)]
+        s = stream or torch.cuda.Stream(device=self.device)
+        cs = torch.cuda.Stream(device=self.device)
+        evs = [torch.cuda.Event() for _ in spans]
+        logits, root, target = inputs.dev["logits"], inputs.dev["root_tok"], inputs.dev["target_tok"]
+        s.wait_stream(torch.cuda.current_stream(self.device))
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=s):
+            cs.wait_stream(s)
+            inputs.upload_head(s)
+            for (a, b), e in zip(spans, evs):
+                inputs.upload_queries(cs, a, b)
+                e.record(cs)
+            self.select(logits, root, ctx_len, s)
+            for (a, b), e in zip(spans, evs):
+                s.wait_event(e)
+                for li in range(a, b):
+                    q, kc, vc, bt = layers[li]
+                    self.verify_layer(q, kc, vc, bt, ctx_len, outs[li], s)
+            self.accept(target, s)
+            s.wait_stream(cs)
+            self.download(host_results, s)
+        torch.cuda.current_stream(self.device).wait_stream(s)
+        return g
+
 
 class RoundInputs:
     """A round's inputs in one device buffer mirrored by one pinned host

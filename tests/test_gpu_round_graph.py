@@ -1,10 +1,10 @@
 """The whole round with its host uploads and the read of its results captured
-as one CUDA graph (the form bench.py's end-to-end figure replays: the head on
-the compute stream, the queries in groups of layers on a copy stream, each
-group of verification layers waiting only for its own), against the same
-round run stage by stage from inputs already on the device. The device copy
-of the inputs is cleared first, so the graph's own uploads must supply them;
-the results must match bit for bit."""
+as one CUDA graph by TapsRound.capture_round_graph (the form bench.py's
+end-to-end figure replays: the head on the compute stream, the queries in
+groups of layers on a copy stream, each group of verification layers waiting
+only for its own), against the same round run stage by stage from inputs
+already on the device. The device copy of the inputs is cleared first, so the
+graph's own uploads must supply them; the results must match bit for bit."""
 import pytest
 
 torch = pytest.importorskip("torch")
@@ -53,3 +53,25 @@ def test_round_graph_with_uploads_matches_stagewise(taps, name, layers, groups):
     g.replay()
     rs.stream.synchronize()
     assert torch.equal(got, expected)
+
+
+def test_round_graph_rejects_unfed_queries(taps):
+    """capture_round_graph refuses a layer whose q is not the upload buffer's
+    view of that layer (the graph's uploads would never reach it) and a result
+    buffer that is not pinned or has the wrong size."""
+    import bench
+    cfg = bench.workload_config("tiny")
+    dev = torch.device("cuda:0")
+    rs = bench.RoundSetup(taps, W, cfg, "taps", dev)
+    r = rs.r
+    res = torch.empty(r.results.shape, dtype=r.results.dtype, pin_memory=True)
+    layers = list(rs.layers)
+    q, kc, vc, bt = layers[0]
+    layers[0] = (q.clone(), kc, vc, bt)
+    with pytest.raises(ValueError):
+        r.capture_round_graph(rs.inp, rs.ctx, layers, rs.outs, res)
+    with pytest.raises(ValueError):
+        r.capture_round_graph(rs.inp, rs.ctx, rs.layers, rs.outs,
+                              torch.empty(r.results.shape, dtype=r.results.dtype))
+    with pytest.raises(ValueError):
+        r.capture_round_graph(rs.inp, rs.ctx, rs.layers[:-1], rs.outs[:-1], res)
