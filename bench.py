@@ -755,7 +755,10 @@ def run_ours(args):
 
 def run_only_topk(args):
     """Stage 1 alone on the workload's logits (for profiling it at a given batch
-    without allocating the KV caches): prints microseconds per call."""
+    without allocating the KV caches): prints microseconds per call, as one call
+    per CUDA graph replay (graph launch included, as in stage_us) and as 20 calls
+    back to back in one graph (each launch overlapping the previous one's tail,
+    as in the round)."""
     import torch
     import __graft_entry__
     __graft_entry__.build()
@@ -764,19 +767,35 @@ def run_only_topk(args):
     cfg = workload_config(args.workload, args.n_max, args.layers, args.mode)
     ldt = torch.bfloat16 if cfg.logits_dtype == "bf16" else torch.float32
     x = torch.from_numpy(W.make_logits(cfg)).to("cuda").to(ldt)
-    for _ in range(args.warmup):
-        taps.taps_topk_marginals(x, cfg.K)
-    torch.cuda.synchronize()
-    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    a.record()
-    for _ in range(args.steps):
-        taps.taps_topk_marginals(x, cfg.K)
-    b.record()
-    torch.cuda.synchronize()
-    us = a.elapsed_time(b) / args.steps * 1e3
+    B, L = x.shape[0], x.shape[1]
+    outs = (torch.empty((B, L, cfg.K), dtype=torch.int32, device="cuda"),
+            torch.empty((B, L, cfg.K), dtype=torch.float32, device="cuda"),
+            torch.empty((B, L), dtype=torch.float32, device="cuda"),
+            torch.empty((B, L), dtype=torch.float32, device="cuda"))
+    ws = torch.zeros(taps.topk_marginals_workspace_bytes(B, L, cfg.V, cfg.K), dtype=torch.uint8,
+                     device="cuda")
+    s = torch.cuda.Stream()
+    res = {}
+    with torch.cuda.stream(s):   # the graphs are replayed, and timed, on s
+        for name, calls in (("us_per_call_one_per_graph", 1), ("us_per_call_back_to_back", 20)):
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=s):
+                for _ in range(calls):
+                    taps.taps_topk_marginals(x, cfg.K, out=outs, ws=ws)
+            for _ in range(args.warmup):
+                g.replay()
+            torch.cuda.synchronize()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(s)
+            for _ in range(args.steps):
+                g.replay()
+            b.record(s)
+            torch.cuda.synchronize()
+            res[name] = round(a.elapsed_time(b) / (args.steps * calls) * 1e3, 2)
     nbytes = x.numel() * x.element_size()
-    print(json.dumps({"stage": "topk_marginals", "workload": cfg.name, "us_per_call": round(us, 2),
-                      "bytes": nbytes, "gbs": round(nbytes / us / 1e3, 1)}), flush=True)
+    print(json.dumps({"stage": "topk_marginals", "workload": cfg.name, **res, "bytes": nbytes,
+                      "gbs_back_to_back": round(nbytes / res["us_per_call_back_to_back"] / 1e3, 1)}),
+          flush=True)
 
 
 def run_reference(args):

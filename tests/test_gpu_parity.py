@@ -113,6 +113,64 @@ def test_topk_value_ties_at_the_threshold(taps, dtype):
     _check_topk(taps, x, 16, dtype)
 
 
+def _padded(x, dtype, mult=8):
+    """x on the device in a row buffer padded to a multiple of `mult`
+    elements, so that rows start on 16-byte boundaries whatever V is (the
+    vector paths, including the one-cluster-per-row kernel for few rows)."""
+    B, L, V = x.shape
+    Vp = -(-V // mult) * mult
+    full = np.zeros((B, L, Vp), np.float32)
+    full[:, :, :V] = x
+    return dt(full).to(dtype)[:, :, :V]
+
+
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
+@pytest.mark.parametrize("V,K,B,L", [(1, 1, 1, 1), (7, 7, 1, 3), (2047, 5, 2, 2), (4099, 32, 1, 2),
+                                     (32000, 4, 1, 8), (100003, 16, 1, 5), (128256, 8, 1, 10),
+                                     (151936, 8, 1, 16), (151937, 1, 1, 16), (262143, 3, 1, 1),
+                                     (151936, 2, 4, 24)])
+def test_topk_few_rows_aligned(taps, V, K, B, L, dtype):
+    """Rows on 16-byte boundaries with few rows: the one-cluster-per-row path
+    (partial vectors at the end of the row, rows shorter than a CTA's slice,
+    every K from 1 to 32, and a shape with too many rows for it)."""
+    rng = np.random.default_rng(V + K)
+    x = (rng.standard_normal((B, L, V)) * 4).astype(np.float32)
+    if dtype == torch.bfloat16:
+        x = W.round_to_bf16(x)
+    _check_topk(taps, x, K, dtype, x_dev=_padded(x, dtype))
+
+
+def test_topk_few_rows_ties_and_minus_inf(taps):
+    rng = np.random.default_rng(5)
+    x = rng.integers(-4, 3, size=(1, 16, 30011)).astype(np.float32)   # heavy exact ties
+    x[0, 0, ::3] = -np.inf
+    x[0, 1, :] = 0.0
+    x[0, 1, 17] = -0.0
+    x[0, 2, :] = -np.inf                                               # 40 finite logits
+    x[0, 2, rng.choice(30011, size=40, replace=False)] = rng.integers(-2, 2, size=40)
+    x[0, 3, 32:] = -np.inf                                             # exactly K finite
+    for dtype in (torch.float32, torch.bfloat16):
+        _check_topk(taps, x, 32, dtype, x_dev=_padded(x, dtype))
+        _check_topk(taps, x, 1, dtype, x_dev=_padded(x, dtype))
+
+
+@pytest.mark.parametrize("K", [16, 32])
+def test_topk_few_rows_many_candidates(taps, K):
+    """Every 256-th 16-byte vector repeats (value falling with the vector index
+    modulo 256): the lanes holding the largest values hold many copies of them,
+    so far more elements than one CTA lists reach the first key threshold and
+    the threshold is raised until they fit. Exact ties everywhere, decided by
+    token id."""
+    V = 151936
+    vec = np.arange(V) // 8
+    x = (-(vec % 256) * 0.125).astype(np.float32)[None, None, :].repeat(16, axis=1)
+    x[0, 1] = x[0, 1][::-1]
+    x[0, 2, ::2] -= 0.0625
+    for dtype in (torch.bfloat16, torch.float32):
+        xd = W.round_to_bf16(x) if dtype == torch.bfloat16 else x
+        _check_topk(taps, xd, K, dtype, x_dev=_padded(xd, dtype))
+
+
 def test_topk_strided_rows(taps):
     """Rows with a stride that is not a multiple of 16 bytes take the scalar path."""
     rng = np.random.default_rng(4)
