@@ -134,7 +134,7 @@ struct Smem {
   static constexpr uint32_t kRecv = kV + kVStages * kTileBytes;
   static constexpr uint32_t kRecvBytes = (152 * (2 * D + 8) + 1023) / 1024 * 1024;
   static constexpr uint32_t kBar = kRecv + kRecvBytes;
-  static constexpr int kNumBars = 2 * kKStages + 2 * kVStages + 2 * kSBufs + 5;
+  static constexpr int kNumBars = kKStages + 2 * kVStages + 2 * kSBufs + 4;
   static constexpr uint32_t kTmemSlot = kBar + 8 * kNumBars;
   static constexpr uint32_t kAbort = kTmemSlot + 4;
   static constexpr uint32_t kMl = (kAbort + 4 + 15) / 16 * 16;   // [128] (max, sum) of the rows
@@ -174,16 +174,18 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
   const uint32_t sb = smem_u32(smem);
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + S::kBar);
   uint64_t* k_full = bars;
-  uint64_t* k_empty = k_full + kKStages;
-  uint64_t* v_full = k_empty + kKStages;
+  uint64_t* v_full = k_full + kKStages;
+  // [kVStages] the burst holding PV of a tile done: V slot free, and O holds
+  // that tile's product (the softmax waits on it before rescaling O)
   uint64_t* v_empty = v_full + kVStages;
-  uint64_t* s_full = v_empty + kVStages;   // [kSBufs] S of a tile written
+  // [kSBufs] QK of a tile done: S written, and its K slot free (the K
+  // producer waits on it too)
+  uint64_t* s_full = v_empty + kVStages;
   // [kSBufs] P of a tile written (4 warps arrive). One per buffer: the
   // softmax may finish tile j+1 before the MMA warp has waited for tile j,
   // and a single barrier would then complete two phases in a row
   uint64_t* p_full = s_full + kSBufs;
-  uint64_t* pv_done = p_full + kSBufs;     // the burst holding PV of a tile done
-  uint64_t* o_full = pv_done + 1;          // last PV done
+  uint64_t* o_full = p_full + kSBufs;      // last PV done
   uint64_t* q_full = o_full + 1;
   uint64_t* drain = q_full + 1;
   uint64_t* recv = drain + 1;              // the peers' partial rows of this CTA's slice landed
@@ -208,10 +210,7 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
   const int re = min(kRowsPerCta, rb + per);
   if (threadIdx.x == 0) {
     prefetch_tensormap(&maps.q);
-    for (int s = 0; s < kKStages; ++s) {
-      mbar_init(&k_full[s], 1);
-      mbar_init(&k_empty[s], 1);
-    }
+    for (int s = 0; s < kKStages; ++s) mbar_init(&k_full[s], 1);
     for (int s = 0; s < kVStages; ++s) {
       mbar_init(&v_full[s], 1);
       mbar_init(&v_empty[s], 1);
@@ -220,7 +219,6 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
       mbar_init(&s_full[u], 1);
       mbar_init(&p_full[u], 4);
     }
-    mbar_init(pv_done, 1);
     mbar_init(o_full, 1);
     mbar_init(q_full, 1);
     mbar_init(drain, 1);
@@ -347,14 +345,18 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
     const bool is_k = warp == 0;
     const int nst = is_k ? kKStages : kVStages;
     uint64_t* full = is_k ? k_full : v_full;
-    uint64_t* empty = is_k ? k_empty : v_empty;
     auto in_chunk = [&](int j) { return lane < kTilePages && pos0 + j * kTile + 16 * lane < pos1; };
     int pg = n_tiles > 1 && in_chunk(1) ? spages[kTilePages + lane] : -1;
     int issued = 1;
     for (int j = 1; j < n_tiles; ++j) {
       if (__any_sync(kFullMask, *abort_flag != 0)) break;
       const int s = j % nst;
-      if (j >= nst && !__all_sync(kFullMask, mbar_wait(&empty[s], ((j / nst) - 1) & 1))) {
+      // slot s last held tile t = j - nst: free once QK (K) or the burst
+      // holding PV (V) of tile t is done. Neither barrier can have completed
+      // its following phase yet: that needs a tile this warp has not issued.
+      const int t = j - nst;
+      if (j >= nst && !__all_sync(kFullMask, is_k ? mbar_wait(&s_full[t % kSBufs], (t / kSBufs) & 1)
+                                                  : mbar_wait(&v_empty[s], (t / kVStages) & 1))) {
         if (lane == 0) set_fault(abort_flag, a.status, TAPS_DEVFAULT_TIMEOUT);
         break;
       }
@@ -387,7 +389,6 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
 #pragma unroll
         for (int ks = 0; ks < kQkSteps; ++ks) qk_step(jj, ks);
         mma_commit(&s_full[jj % kSBufs]);
-        mma_commit(&k_empty[jj % kKStages]);
       }
       __syncwarp();
     }
@@ -463,12 +464,9 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
           }
           if (has_qk && ks < kQkSteps) qk_step(jn, ks);
         }
-        mma_commit(pv_done);
+        // S first: the softmax waits on it; then the V slot / O update
+        if (has_qk) mma_commit(&s_full[jn % kSBufs]);
         mma_commit(&v_empty[sv]);
-        if (has_qk) {
-          mma_commit(&s_full[jn % kSBufs]);
-          mma_commit(&k_empty[jn % kKStages]);
-        }
         if (j == n_tiles - 1) mma_commit(o_full);
       }
       __syncwarp();
@@ -609,7 +607,8 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
       // the previous tile may still be running, so wait for it first
       const bool need_rescale = grow_max && j > 0 && alpha != 1.f;
       if (__any_sync(kFullMask, need_rescale)) {
-        if (!__all_sync(kFullMask, mbar_wait(pv_done, (j - 1) & 1))) {
+        if (!__all_sync(kFullMask, mbar_wait(&v_empty[(j - 1) % kVStages],
+                                             ((j - 1) / kVStages) & 1))) {
           if (lane == 0) set_fault(abort_flag, a.status, TAPS_DEVFAULT_TIMEOUT);
           ok = false;
           break;
