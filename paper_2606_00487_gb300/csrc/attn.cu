@@ -748,34 +748,47 @@ attn_tc_kernel(const __grid_constant__ Maps maps, const Args a) {
   }
   __syncthreads();
   if (got) {
-    for (int e = threadIdx.x; e < (re - rb) * (D / 8); e += kThreadsTc) {
-      const int i = e / (D / 8), q16 = e % (D / 8);
+    // kTpr threads per row, each combining two adjacent 16-byte pieces of it,
+    // so that the row's output offset, statistics and reciprocal are worked
+    // out once per row rather than once per piece
+    constexpr int kTpr = D / 16;
+    constexpr int kRowsPerPass = kThreadsTc / kTpr;
+    const int qa = 2 * (threadIdx.x % kTpr);        // pieces qa, qa + 1 of the row's D / 8
+    for (int i = threadIdx.x / kTpr; i < re - rb; i += kRowsPerPass) {
       const int rr = rb + i, gr = row0 + rr;
       if (gr >= pl.rows_max) continue;
-      const uint8_t* vp = rv + ((q16 >> 3) * per + i) * 128 + (((q16 & 7) ^ (rr & 7)) << 4);
-      float acc[8];
-#pragma unroll
-      for (int k = 0; k < 8; ++k) acc[k] = 0.f;
-#pragma unroll 4
-      for (int q = 0; q < cs; ++q) {
-        const float w = rml[q * per + i].x;
-        const uint4 v = *reinterpret_cast<const uint4*>(vp + q * CH * per * 128);
-        const uint32_t u[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          acc[2 * k] = fmaf(w, __uint_as_float(u[k] << 16), acc[2 * k]);
-          acc[2 * k + 1] = fmaf(w, __uint_as_float(u[k] & 0xFFFF0000u), acc[2 * k + 1]);
-        }
-      }
       const float2 st = stat[i];
       const bool row_ok = gr < rows && st.y > 0.f;
       const float linv = row_ok ? 1.f / st.y : 0.f;
       const int64_t orow = (static_cast<int64_t>(b) * a.n_max + gr / pl.group) * a.Hq +
                            kv * pl.group + gr % pl.group;
-      *reinterpret_cast<uint4*>(a.out + orow * D + q16 * 8) = make_uint4(
+      const uint8_t* vp = rv + ((qa >> 3) * per + i) * 128;
+      const uint32_t oa = ((qa & 7) ^ (rr & 7)) << 4, ob = (((qa + 1) & 7) ^ (rr & 7)) << 4;
+      float acc[16];
+#pragma unroll
+      for (int k = 0; k < 16; ++k) acc[k] = 0.f;
+#pragma unroll 4
+      for (int q = 0; q < cs; ++q) {
+        const float w = rml[q * per + i].x;
+        const uint8_t* vq = vp + q * CH * per * 128;
+        const uint4 x = *reinterpret_cast<const uint4*>(vq + oa);
+        const uint4 y = *reinterpret_cast<const uint4*>(vq + ob);
+        const uint32_t u[8] = {x.x, x.y, x.z, x.w, y.x, y.y, y.z, y.w};
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          acc[2 * k] = fmaf(w, __uint_as_float(u[k] << 16), acc[2 * k]);
+          acc[2 * k + 1] = fmaf(w, __uint_as_float(u[k] & 0xFFFF0000u), acc[2 * k + 1]);
+        }
+      }
+      uint4* dst = reinterpret_cast<uint4*>(a.out + orow * D + qa * 8);
+      dst[0] = make_uint4(
           pack_bf16x2(acc[0] * linv, acc[1] * linv), pack_bf16x2(acc[2] * linv, acc[3] * linv),
           pack_bf16x2(acc[4] * linv, acc[5] * linv), pack_bf16x2(acc[6] * linv, acc[7] * linv));
-      if (a.lse && q16 == 0) a.lse[orow] = row_ok ? (st.x + log2f(st.y)) * kLn2 : 0.f;
+      dst[1] = make_uint4(
+          pack_bf16x2(acc[8] * linv, acc[9] * linv), pack_bf16x2(acc[10] * linv, acc[11] * linv),
+          pack_bf16x2(acc[12] * linv, acc[13] * linv),
+          pack_bf16x2(acc[14] * linv, acc[15] * linv));
+      if (a.lse && qa == 0) a.lse[orow] = row_ok ? (st.x + log2f(st.y)) * kLn2 : 0.f;
     }
   }
   // every peer has received what this CTA sent it before this CTA exits
