@@ -165,6 +165,11 @@ int taps_topk_marginals_noalloc(const void* logits, int dtype, int64_t row_strid
  *                        device f32 buffer: tok_emb[vocab][E], dep_emb[max_depth][E],
  *                        W1[H][3E+2], b1[H], w2[H], w_lp[1], packed in that
  *                        order. Token ids must be < vocab; max_depth > L.
+ *                        The kernel stages W1, b1, w2, w_lp and the depth
+ *                        embeddings before it waits for the kernel launched
+ *                        just before it on `stream` (programmatic dependent
+ *                        launch), so that kernel must not write them (none
+ *                        of this library's kernels does).
  *
  * Reach of an explicit node list (Eq. 2), optional: paths, path_len and
  * path_reach are all NULL with M == 0, or all given with M >= 1.

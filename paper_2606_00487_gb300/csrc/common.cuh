@@ -21,10 +21,11 @@ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 // Programmatic dependent launch. Every kernel of the library is launched
 // with programmatic stream serialisation, so that its launch and prologue may
-// overlap the tail of the kernel before it on the stream. dep_enter() is the
-// first statement of every such kernel: it waits until the previous grid has
-// completed and its memory is visible (so no input is read and no output
-// written before that), then lets the next kernel on the stream be launched.
+// overlap the tail of the kernel before it on the stream. dep_enter() comes
+// before every read of an input another kernel may write and before every
+// output write (it is the first statement of most kernels; the scorer stages
+// its weights ahead of it): it waits until the previous grid has completed and
+// its memory is visible, then lets the next kernel on the stream be launched.
 __device__ __forceinline__ void dep_enter() {
   asm volatile("griddepcontrol.wait;" ::: "memory");
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");

@@ -21,7 +21,6 @@ score_kernel(const int32_t* __restrict__ root_tok, const int32_t* __restrict__ i
              const float* __restrict__ logp, const float* __restrict__ entropy, int L, int K,
              int kind, int E, int H, int vocab, int max_depth, const float* __restrict__ w,
              float* __restrict__ q_cond) {
-  dep_enter();
   extern __shared__ float sm[];
   const int d = blockIdx.x;
   const int b = blockIdx.y;
@@ -55,16 +54,20 @@ score_kernel(const int32_t* __restrict__ root_tok, const int32_t* __restrict__ i
   const float* W1 = dep_emb + static_cast<int64_t>(max_depth) * E;
   const float* b1 = W1 + H * F;
   const float* w2 = b1 + H;
-  for (int j = tid; j < K; j += kThreads) {
-    s_logp[j] = logp[row0 + j];
-    s_ctok[j] = ids[row0 + j];
-    s_ptok[j] = d == 0 ? root_tok[b] : ids[row0 - K + j];
-  }
+  // The MLP's weights are no output of any kernel of the round: they are
+  // staged before the wait for the preceding grid, overlapping its tail
+  // (the caller's contract, include/taps.h).
   if (mlp) {
     for (int i = tid; i < H * F; i += kThreads) s_W1[(i / F) * FP + i % F] = W1[i];
     for (int i = tid; i < 2 * H + 1; i += kThreads) s_b1[i] = b1[i];   // b1, then w2 and its logp weight
     const float* drow = dep_emb + static_cast<int64_t>(min(d + 1, max_depth - 1)) * E;
     for (int i = tid; i < E; i += kThreads) s_dep[i] = drow[i];
+  }
+  dep_enter();
+  for (int j = tid; j < K; j += kThreads) {
+    s_logp[j] = logp[row0 + j];
+    s_ctok[j] = ids[row0 + j];
+    s_ptok[j] = d == 0 ? root_tok[b] : ids[row0 - K + j];
   }
   __syncthreads();
 
