@@ -21,7 +21,7 @@ BUILD = os.path.join(PKG, "_build")
 LIBDIR = os.path.join(PKG, "_lib")
 LIB = os.path.join(LIBDIR, "libtaps.so")
 
-SOURCES = ["api.cu", "topk.cu", "topk_cluster.cu", "score.cu", "select.cu", "mask.cu", "attn.cu", "accept.cu",
+SOURCES = ["api.cu", "topk.cu", "topk_cluster.cu", "topk_stream.cu", "score.cu", "select.cu", "mask.cu", "attn.cu", "accept.cu",
            "kvpack.cu", "target.cu", "compact.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",

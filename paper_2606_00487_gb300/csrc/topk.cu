@@ -557,6 +557,10 @@ extern "C" int taps_topk_marginals(const void* logits, int dtype, int64_t row_st
   const int rc = topk_cluster_try(logits, dtype, row_stride, B * L, V, K, topk_ids, topk_logp, lse,
                                   entropy, s);
   if (rc != -1) return rc;
+  // many rows: one CTA streams each row
+  const int rs = topk_stream_try(logits, dtype, row_stride, B * L, V, K, topk_ids, topk_logp, lse,
+                                 entropy, s);
+  if (rs != -1) return rs;
   const size_t esz = dtype == TAPS_F32 ? 4 : 2;
   const int vec_ok = aligned(logits, 16) && (row_stride * esz) % 16 == 0;
   char* wsc = static_cast<char*>(ws);

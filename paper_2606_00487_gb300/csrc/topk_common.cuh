@@ -12,6 +12,10 @@ namespace taps {
 // (nothing launched) when the shape is left to topk_marginals_kernel.
 int topk_cluster_try(const void* logits, int dtype, int64_t row_stride, int R, int V, int K,
                      int32_t* ids, float* logp, float* lse, float* ent, cudaStream_t s);
+// Stage 1 for many rows (topk_stream.cu): one CTA streams one row. Same
+// return convention.
+int topk_stream_try(const void* logits, int dtype, int64_t row_stride, int R, int V, int K,
+                    int32_t* ids, float* logp, float* lse, float* ent, cudaStream_t s);
 
 namespace {
 

@@ -171,6 +171,39 @@ def test_topk_few_rows_many_candidates(taps, K):
         _check_topk(taps, xd, K, dtype, x_dev=_padded(xd, dtype))
 
 
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
+@pytest.mark.parametrize("V,K", [(30011, 8), (65539, 32), (4093, 1), (151936, 16)])
+def test_topk_many_rows(taps, V, K, dtype):
+    """320 rows (20 requests x 16 positions): one CTA streams each row
+    (partial last stage, the elements after the last whole vector, K from 1
+    to 32)."""
+    rng = np.random.default_rng(V + 7 * K)
+    x = (rng.standard_normal((20, 16, V)) * 3).astype(np.float32)
+    if dtype == torch.bfloat16:
+        x = W.round_to_bf16(x)
+    _check_topk(taps, x, K, dtype, x_dev=_padded(x, dtype))
+
+
+def test_topk_many_rows_ties_and_special_rows(taps):
+    """320 rows of heavy exact ties (small integers), so the first threshold's
+    value is shared by thousands of elements and a stage overflows the
+    candidate list; plus rows of one value, rows mostly -inf, and rows whose
+    16-byte vectors repeat every 256 vectors."""
+    rng = np.random.default_rng(11)
+    V = 20011
+    x = rng.integers(-3, 3, size=(20, 16, V)).astype(np.float32)
+    x[0, 0, :] = 1.5                                                   # one value
+    x[0, 1, :] = -np.inf
+    x[0, 1, rng.choice(V, size=40, replace=False)] = rng.integers(-2, 2, size=40)
+    x[0, 2, ::2] = -np.inf
+    vec = np.arange(V) // 8
+    x[1, 0] = -(vec % 256) * 0.125                                     # periodic vectors
+    x[1, 1] = x[1, 0][::-1]
+    for dtype in (torch.float32, torch.bfloat16):
+        for K in (32, 8, 1):
+            _check_topk(taps, x, K, dtype, x_dev=_padded(x, dtype))
+
+
 def test_topk_strided_rows(taps):
     """Rows with a stride that is not a multiple of 16 bytes take the scalar path."""
     rng = np.random.default_rng(4)
