@@ -110,7 +110,7 @@ topk_cluster_kernel(const T* __restrict__ logits, int64_t row_stride, int V, int
   __shared__ uint64_t s_part[kClWarps * KP];
   __shared__ uint64_t s_ckeys[kClMaxCluster * KP];    // [CTA][KP], written by the cluster's CTAs
   __shared__ float4 s_cst[kClMaxCluster];             // [CTA] statistics (m2, z, t2)
-  __shared__ float s_vmax[kClMaxNv * kClThreads];       // [vector i][thread] maxima
+  __shared__ float s_vmax[kClMaxNv * kClThreads];     // [vector i][thread] maxima
   __shared__ Stats s_wst[kClWarps];
   __shared__ __align__(8) uint64_t s_bar;             // the slice's copies landed
   __shared__ unsigned s_vthr;   // ordered value that at least KP elements of the slice reach
