@@ -725,8 +725,12 @@ def test_kv_pack_layout(taps, D):
 # Stage 6
 # ---------------------------------------------------------------------------
 
+@pytest.mark.parametrize("per_node", [False, True])
 @pytest.mark.parametrize("seed", range(6))
-def test_accept_parity(taps, seed):
+def test_accept_parity(taps, seed, per_node):
+    """Target tokens either follow one target sequence (a function of depth)
+    or are drawn per node (nodes of one depth want different tokens, as their
+    prefixes differ)."""
     rng = np.random.default_rng(seed)
     B, L, K, n_max = 4, 16, 4, 96
     raw = rng.random((B, L, K, K)) + 0.05
@@ -740,6 +744,10 @@ def test_accept_parity(taps, seed):
                            n_max)
     y = rng.integers(0, 6, size=(B, L + 1)).astype(np.int32)
     tt = W.target_tokens_for_tree(y, sel["depth"], sel["n_nodes"])
+    if per_node:
+        for b in range(B):
+            n = int(sel["n_nodes"][b])
+            tt[b, :n] = rng.integers(0, 6, size=n)
     alen, nodes, bonus = taps.taps_accept(dt(sel["parent"]), dt(sel["token"]),
                                           dt(sel["n_nodes"]), dt(tt), L)
     torch.cuda.synchronize()

@@ -219,6 +219,31 @@ def test_depth_embedding_index_is_edge_depth():
             assert diff < 1e-6
 
 
+def test_entropy_feature_is_the_child_position():
+    """E=1, H=1: relu(E_tok[child] + H) with a different entropy H at each
+    position. Position d's rows are then softmax(relu(e_child + H[d])) over
+    the siblings, a closed form that fixes which position's entropy enters."""
+    L = 3
+    ids = np.array([[[0, 1, 2]] * L], np.int32)
+    e = np.array([0.0, -1.0, -2.0])
+    tok = np.zeros((50, 1), F32)
+    tok[:3, 0] = e
+    ent = np.array([[0.0, 1.5, 3.0]])
+    W1 = np.zeros((1, 3 * 1 + 2), F32)
+    W1[0, 1] = 1.0          # child embedding
+    W1[0, 4] = 1.0          # positional entropy
+    w = _weights(50, L, 1, 1, tok_emb=tok, W1=W1, b1=np.zeros(1, F32),
+                 w2=np.array([1.0], F32), w_lp=np.array([0.0], F32))
+    q = O.score_qcond(np.array([7]), ids, np.zeros((1, L, 3)), ent, kind="mlp", weights=w)
+    for d in range(L):
+        h = np.maximum(e + ent[0, d], 0.0)
+        expect = np.exp(h) / np.exp(h).sum()
+        rows = [0] if d == 0 else range(3)
+        for i in rows:
+            np.testing.assert_allclose(q[0, d, i], expect, rtol=1e-6)
+    assert np.abs(q[0, 1, 0] - q[0, 2, 0]).max() > 1e-2     # the positions do differ
+
+
 def test_parent_token_enters_through_interaction():
     """E=1, H=1: relu(E_tok[parent] + E_tok[child] - 5) is non-zero only under
     one chosen parent token; rows of other parents equal the marginal."""
@@ -623,6 +648,28 @@ def test_attention_zero_query_is_mean_of_visible_values():
             assert lse[0, i, h] == pytest.approx(math.log(len(pos)), rel=1e-12)
 
 
+def test_attention_identical_keys_closed_form():
+    """Every key of a KV head is the same vector k_h: all visible scores of a
+    query equal s = q.k_h / sqrt(D), so the softmax is uniform (the output is
+    the mean of the visible values) and lse = s + log(number visible)."""
+    q, k, v, bt, ctx, nn, mask = _attn_case(6, 5, parents=[-1, 0, 0, 1, 3])
+    rng = np.random.default_rng(60)
+    kvec = rng.standard_normal((k.shape[1], k.shape[3]))
+    k = np.broadcast_to(kvec[None, :, None, :], k.shape).copy()
+    q = 3.0 * q
+    out, lse = O.tree_verify_attn(q, k, v, bt, ctx, nn, mask)
+    C, P, D = int(ctx[0]), k.shape[2], k.shape[3]
+    anc = {0: [0], 1: [0, 1], 2: [0, 2], 3: [0, 1, 3], 4: [0, 1, 3, 4]}
+    for i, a in anc.items():
+        pos = list(range(C)) + [C + j for j in a]
+        for h in range(4):
+            s = float(q[0, i, h] @ kvec[h // 2]) / math.sqrt(D)
+            assert abs(s) > 0.1
+            assert lse[0, i, h] == pytest.approx(s + math.log(len(pos)), rel=1e-12, abs=1e-12)
+            rows = np.stack([v[bt[0, t // P], h // 2, t % P] for t in pos])
+            np.testing.assert_allclose(out[0, i, h], rows.mean(0), rtol=1e-10, atol=1e-12)
+
+
 def test_attention_page_placement_invariance():
     q, k, v, bt, ctx, nn, mask = _attn_case(5, 7)
     out1, _ = O.tree_verify_attn(q, k, v, bt, ctx, nn, mask)
@@ -674,6 +721,30 @@ def test_accept_brute_force(seed):
     # accepted draft tokens + bonus = the target's greedy continuation
     toks = [int(s["token"][0, v]) for v in nodes[0, 1:alen[0] + 1]] + [int(bonus[0])]
     assert toks == y[0, :alen[0] + 1].tolist()
+
+
+@pytest.mark.parametrize("seed", range(8))
+def test_accept_brute_force_per_node_targets(seed):
+    """The target's greedy token at a node depends on the node's whole prefix,
+    so two nodes of the same depth can want different tokens: random target
+    tokens per node, checked against brute force over root paths."""
+    rng = np.random.default_rng(450 + seed)
+    L, K, A, n_max = 5, 3, 4, 40
+    q = _random_qcond(rng, L, K)[None]
+    ids = np.stack([rng.permutation(A)[:K] for _ in range(L)]).astype(np.int32)[None]
+    s = O.select_subtree(q, ids, np.array([0]), np.array([0]), 1.0, 0.1, 0.0, n_max)
+    n = int(s["n_nodes"][0])
+    tt = np.full((1, n_max), -1, np.int32)
+    tt[0, :n] = rng.integers(0, A, size=n)
+    alen, nodes, bonus = O.accept(s["parent"], s["token"], s["n_nodes"], tt, L)
+    last = _brute_force_accept(s["parent"][0], s["token"][0], n, tt[0])
+    chain = [last]
+    while chain[-1] != 0:
+        chain.append(int(s["parent"][0, chain[-1]]))
+    assert alen[0] == len(chain) - 1
+    assert nodes[0, :len(chain)].tolist() == chain[::-1]
+    assert np.all(nodes[0, len(chain):] == -1)
+    assert bonus[0] == tt[0, last]
 
 
 def test_accept_chain_is_longest_prefix_match():
