@@ -152,11 +152,14 @@ class ClockSampler:
 # CPU baseline: the oracle as it stands, on a bounded sample of the workload
 # ---------------------------------------------------------------------------
 
-def oracle_step(cfg, inp, sample_layers, kind="mlp", pool=None):
+def oracle_step(cfg, inp, sample_layers, kind="mlp", pool=None, pairs=None):
     """One oracle round: stages 1-4 and 6 on the whole batch, stage 5 on
     ``sample_layers`` of the cfg.layers layers; returns seconds scaled to the
     full round. With ``pool`` (worker processes holding the same inputs), each
-    sampled layer's stage 5 is split over the workers by (request, head)."""
+    sampled layer's stage 5 is split over the workers by (request, head).
+    With ``pairs`` (a list of (request, query head)), each sampled layer's
+    stage 5 computes only those pairs' rows, and its time is scaled by the
+    number of pairs in a layer over the number sampled."""
     from oracle import taps_oracle as O
     t0 = time.perf_counter()
     ids, logp, lse, ent = O.topk_marginals(inp["logits"], cfg.K)
@@ -178,11 +181,16 @@ def oracle_step(cfg, inp, sample_layers, kind="mlp", pool=None):
             sum(pool.map(_attn_worker_rows, tasks, chunksize=1))
         t2 = time.perf_counter()
     else:
+        only = None
+        if pairs is not None:
+            only = {(b, i, h) for (b, h) in pairs for i in range(int(sel["n_nodes"][b]))}
         for _ in range(sample_layers):
             O.tree_verify_attn(inp["q"], inp["k"], inp["v"], inp["bt"], inp["ctx"],
-                               sel["n_nodes"], mask)
+                               sel["n_nodes"], mask, only=only)
         t2 = time.perf_counter()
     per_layer = (t2 - t1) / max(sample_layers, 1)
+    if pairs is not None and pool is None:
+        per_layer *= cfg.B * cfg.Hq / len(pairs)
     return (t1 - t0) + cfg.layers * per_layer, t2 - t0
 
 
@@ -242,11 +250,21 @@ def cpu_child(args):
                                             initargs=(cfg,))
         assert all(pool.map(_attn_worker_ready, range(4 * args.cpu_cores), chunksize=1))
     steps, warm = args.steps, args.warmup
-    for _ in range(warm):
-        oracle_step(cfg, inp, args.sample_layers, kind, pool)
+    # with --attn-pairs n, step t samples n (request, head) pairs of a layer,
+    # taken in turn from the list of all pairs so that the steps cover them evenly
+    all_pairs = [(b, h) for b in range(cfg.B) for h in range(cfg.Hq)]
+
+    def pairs_of(t):
+        n = args.attn_pairs
+        if n <= 0 or n >= len(all_pairs):
+            return None
+        return [all_pairs[(t * n + k) % len(all_pairs)] for k in range(n)]
+
+    for t in range(warm):
+        oracle_step(cfg, inp, args.sample_layers, kind, pool, pairs_of(t))
     scaled, wall = [], []
-    for _ in range(steps):
-        s, w = oracle_step(cfg, inp, args.sample_layers, kind, pool)
+    for t in range(steps):
+        s, w = oracle_step(cfg, inp, args.sample_layers, kind, pool, pairs_of(warm + t))
         scaled.append(s)
         wall.append(w)
     if pool is not None:
@@ -255,7 +273,7 @@ def cpu_child(args):
     print(json.dumps({"scaled_s": scaled, "wall_s": wall, "cores": args.cpu_cores}))
 
 
-def run_cpu_baseline(args, steps, warmup, sample_layers, cores=1):
+def run_cpu_baseline(args, steps, warmup, sample_layers, cores=1, attn_pairs=0):
     cfg = workload_config(args.workload, args.n_max, args.layers, args.mode)
     env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1",
                CUDA_VISIBLE_DEVICES="")
@@ -263,16 +281,37 @@ def run_cpu_baseline(args, steps, warmup, sample_layers, cores=1):
            "--mode", args.mode,
            "--n-max", str(cfg.n_max), "--layers", str(cfg.layers), "--steps", str(steps),
            "--warmup", str(warmup), "--sample-layers", str(sample_layers),
-           "--cpu-cores", str(cores)]
+           "--cpu-cores", str(cores), "--attn-pairs", str(attn_pairs)]
     r = subprocess.run(cmd, env=env, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"cpu baseline child failed:\n{r.stderr[-2000:]}")
     return json.loads(r.stdout.strip().splitlines()[-1])
 
 
-def sample_desc(cfg, sample_layers):
+def sample_desc(cfg, sample_layers, attn_pairs=0):
+    if 0 < attn_pairs < cfg.B * cfg.Hq:
+        return (f"oracle stages 1-4 and 6 on the whole round, stage 5 on {attn_pairs} of the "
+                f"{cfg.B * cfg.Hq} (request, query head) pairs of one layer, taken in turn "
+                f"(timed, then scaled to {cfg.layers} whole layers)")
     return (f"oracle stages 1-4 and 6 on the whole round, stage 5 on {sample_layers} of "
             f"{cfg.layers} layers (timed, then scaled to {cfg.layers} layers)")
+
+
+# the reference arm's stage-5 sample: a whole layer per step while the run has at
+# most this many steps (warm-up included), otherwise a share of a layer's pairs
+# sized to keep the run to about as many layers in all; never fewer than 4 pairs
+# (below that, the per-request gathers of K and V outweigh the sampled rows and
+# the scaled time overstates a layer)
+REF_LAYER_BUDGET = 30
+REF_MIN_PAIRS = 4
+
+
+def reference_attn_pairs(cfg, steps, warmup):
+    total = cfg.B * cfg.Hq
+    n = steps + warmup
+    if n <= REF_LAYER_BUDGET:
+        return 0
+    return min(total, max(REF_MIN_PAIRS, total * REF_LAYER_BUDGET // n))
 
 
 # ---------------------------------------------------------------------------
@@ -805,7 +844,9 @@ def run_reference(args):
     if rank != 0:
         return
     cfg = workload_config(args.workload, args.n_max, args.layers, args.mode)
-    cb = run_cpu_baseline(args, steps=args.steps, warmup=args.warmup, sample_layers=1)
+    pairs = reference_attn_pairs(cfg, args.steps, args.warmup)
+    cb = run_cpu_baseline(args, steps=args.steps, warmup=args.warmup, sample_layers=1,
+                          attn_pairs=pairs)
     total = sum(cb["scaled_s"])
     value = args.steps / total
     line = {
@@ -822,7 +863,7 @@ def run_reference(args):
                    "global_batch": cfg.B, "seq_len": cfg.ctx if isinstance(cfg.ctx, int) else None,
                    "parallelism": "none (host CPU)"},
         "cpu_baseline": {"value": round(value, 5), "unit": "rounds/s", "cores": 1,
-                         "kind": "oracle", "sample": sample_desc(cfg, 1) + " per step"},
+                         "kind": "oracle", "sample": sample_desc(cfg, 1, pairs) + " per step"},
         "e2e": {"value": round(value, 5), "unit": "rounds/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }
@@ -846,6 +887,7 @@ def main():
     ap.add_argument("--no-sweep", action="store_true",
                     help="skip the other configurations (budget sweep, Qwen3-4B, batch 32, long)")
     ap.add_argument("--cpu-cores", type=int, default=1, help=argparse.SUPPRESS)
+    ap.add_argument("--attn-pairs", type=int, default=0, help=argparse.SUPPRESS)
     ap.add_argument("--only-topk", action="store_true",
                     help="time stage 1 alone on the workload's logits (profiling aid)")
     ap.add_argument("--no-cpu-baseline", action="store_true")

@@ -100,3 +100,47 @@ def test_roofline_names_the_binding_bound():
         assert rl["bound"] == bound
         assert rl["avg_launch_us"] == 10.0
         assert abs(rl["hbm_frac"] - rl["algorithmic_bytes_per_launch"] / 10e-6 / 1e9 / 6704.5) < 1e-4
+
+
+def test_reference_arm_sample_size():
+    """The reference arm times a whole layer of stage 5 per step while the run is
+    short, otherwise a share of a layer's (request, head) pairs that keeps the run
+    to about the same number of layers, never below the floor of pairs."""
+    cfg = W.CONFIGS["qwen3_8b"]
+    total = cfg.B * cfg.Hq
+    assert bench.reference_attn_pairs(cfg, 20, 5) == 0
+    assert bench.reference_attn_pairs(cfg, bench.REF_LAYER_BUDGET - 3, 3) == 0
+    for steps in (40, 100, 200, 5000):
+        n = bench.reference_attn_pairs(cfg, steps, 5)
+        assert bench.REF_MIN_PAIRS <= n < total
+        assert n == max(bench.REF_MIN_PAIRS, total * bench.REF_LAYER_BUDGET // (steps + 5))
+    assert "4 of the 32" in bench.sample_desc(cfg, 1, 4)
+    assert "1 of 36 layers" in bench.sample_desc(cfg, 1, 0)
+
+
+def test_oracle_step_pair_sample_covers_the_sampled_rows():
+    """A stage-5 sample of some (request, head) pairs computes exactly those pairs'
+    rows of the layer (the same values as the whole layer there, zeros elsewhere)."""
+    cfg = W.CONFIGS["tiny"].with_(B=2)
+    inp = bench.oracle_attn_inputs(cfg)
+    rng = np.random.default_rng(9)
+    n_nodes = np.array([16, 5], np.int32)
+    parent = np.full((2, 16), -1, np.int32)
+    for b in range(2):
+        for i in range(1, n_nodes[b]):
+            parent[b, i] = rng.integers(0, i)
+    mask = O.build_tree_mask(parent, n_nodes, 16)
+    ref, _ = O.tree_verify_attn(inp["q"], inp["k"], inp["v"], inp["bt"], inp["ctx"], n_nodes, mask)
+    pairs = [(0, 3), (1, 0), (1, 5)]
+    only = {(b, i, h) for (b, h) in pairs for i in range(int(n_nodes[b]))}
+    got, _ = O.tree_verify_attn(inp["q"], inp["k"], inp["v"], inp["bt"], inp["ctx"], n_nodes, mask,
+                                only=only)
+    keep = np.zeros(ref.shape, bool)
+    for b, h in pairs:
+        keep[b, :, h] = True
+    assert np.array_equal(got[keep], ref[keep])
+    assert not got[~keep].any()
+    # and the timed step runs with such a sample (time scaled to whole layers)
+    full = bench.oracle_inputs(cfg)
+    scaled, wall = bench.oracle_step(cfg, full, 1, "mlp", None, pairs)
+    assert scaled > 0 and wall > 0
