@@ -42,6 +42,10 @@ MUTANTS = [
     ("topk_marginals", "child log-probability taken against the maximum, not lse",
      "logp = np.take_along_axis(x, ids.astype(np.int64), axis=-1) - lse[..., None]",
      "logp = np.take_along_axis(x, ids.astype(np.int64), axis=-1) - m[..., None]"),
+    ("topk_marginals", "entropy weighted by unnormalised probabilities",
+     "p = np.exp(x - lse[..., None])", "p = np.exp(x - m[..., None])"),
+    ("topk_marginals", "top-K list starting one rank down",
+     "ids[b, d] = order[:K]", "ids[b, d] = order[1:K + 1]"),
     # Stage 2: scorer and sibling softmax (Sec. 4.2, Eq. 1)
     ("edge_logit_mlp", "parent and child embeddings swapped",
      'w["tok_emb"][parent_tok].astype(np.float64),\n        w["tok_emb"][child_tok]',
@@ -57,6 +61,10 @@ MUTANTS = [
     ("edge_logit_mlp", "direct log-probability term dropped",
      'return float(w["w_lp"][0]) * logp_child + float(w["w2"].astype(np.float64) @ h)',
      'return float(w["w2"].astype(np.float64) @ h)'),
+    ("edge_logit_mlp", "depth embedding of the parent's depth",
+     'w["dep_emb"][depth].astype(np.float64)', 'w["dep_emb"][depth - 1].astype(np.float64)'),
+    ("edge_logit_mlp", "direct term multiplies the entropy",
+     'return float(w["w_lp"][0]) * logp_child +', 'return float(w["w_lp"][0]) * entropy +'),
     ("score_qcond", "edge depth off by one (position index used)",
      "edge_logit_mlp(weights, ptok, int(ids[b, d, j]), d + 1,",
      "edge_logit_mlp(weights, ptok, int(ids[b, d, j]), d,"),
@@ -74,6 +82,11 @@ MUTANTS = [
     # Eq. 2: reach
     ("reach_of_path", "q_cond indexed [child, parent]",
      "r *= float(q_cond_b[d, parent_slot, j])", "r *= float(q_cond_b[d, j, parent_slot])"),
+    ("reach_of_path", "q_cond summed instead of multiplied",
+     "r *= float(q_cond_b[d, parent_slot, j])", "r += float(q_cond_b[d, parent_slot, j])"),
+    ("reach_of_path", "every edge read from the root's row",
+     "        r *= float(q_cond_b[d, parent_slot, j])\n        parent_slot = j",
+     "        r *= float(q_cond_b[d, parent_slot, j])\n        parent_slot = 0"),
     ("path_reach", "q_cond indexed [child, parent]",
      "r = F32(r * F32(q_cond[b, d, parent_slot, j]))",
      "r = F32(r * F32(q_cond[b, d, j, parent_slot]))"),
@@ -82,6 +95,8 @@ MUTANTS = [
      "            r = F32(r * F32(q_cond[b, d, parent_slot, j]))\n                parent_slot = 0"),
     ("path_reach", "full-length paths treated as outside the trie",
      "if n < 0 or n > L or any(j >= K for j in slots):", "if n < 0 or n >= L or any(j >= K for j in slots):"),
+    ("path_reach", "the root treated as outside the trie",
+     "if n < 0 or n > L or any(j >= K for j in slots):", "if n <= 0 or n > L or any(j >= K for j in slots):"),
     # Eq. 3 and Algorithm 1
     ("utility_denominators", "cost term counted one level deeper",
      "F32(l1 + F32(l2 * F32(d)))", "F32(l1 + F32(l2 * F32(d + 1)))"),
@@ -108,6 +123,13 @@ MUTANTS = [
      'if u["depth"] == L:\n                    continue', 'if u["depth"] == L - 1:\n                    continue'),
     ("select_subtree", "budget counted without the root",
      "        while len(S) < n_max:\n            best = None", "        while len(S) < n_max - 1:\n            best = None"),
+    ("select_subtree", "root utility without its denominator",
+     "reach=F32(1.0),\n                    utility=F32(F32(1.0) / den[0]))\n        S = [root]",
+     "reach=F32(1.0),\n                    utility=F32(1.0))\n        S = [root]"),
+    ("select_subtree", "reach carried in double precision (a different rounding)",
+     'r = F32(u["reach"] * q_cond[b, d, prow, j])', 'r = float(u["reach"]) * float(q_cond[b, d, prow, j])'),
+    ("select_subtree", "slot output holds the token",
+     'out["slot"][b, i] = v["slot"]', 'out["slot"][b, i] = v["token"]'),
     ("materialise_trie", "every child read from the root's q_cond row",
      "prow = 0 if d == 0 else path[-1]", "prow = 0"),
     # Stage 4: ancestor mask
@@ -132,11 +154,19 @@ MUTANTS = [
      "visible[:C] = True", "visible[:max(C - 1, 0)] = True"),
     ("tree_verify_attn", "lse without the maximum",
      "lse[b, i, h] = m + math.log(e.sum())", "lse[b, i, h] = math.log(e.sum())"),
+    ("tree_verify_attn", "values read from the key cache",
+     "out[b, i, h] = (e @ Vb[visible, kv, :]) / e.sum()", "out[b, i, h] = (e @ Kb[visible, kv, :]) / e.sum()"),
+    ("tree_verify_attn", "output not normalised",
+     "out[b, i, h] = (e @ Vb[visible, kv, :]) / e.sum()", "out[b, i, h] = e @ Vb[visible, kv, :]"),
+    ("tree_verify_attn", "tree positions not offset by the context length",
+     "visible[C + j] = True", "visible[j] = True"),
     # Stage 6: acceptance and the target's greedy tokens
     ("accept", "target token looked up by depth instead of by node",
      "want = int(target_tok[b, v])", "want = int(target_tok[b, len(path) - 1])"),
     ("accept", "bonus token taken from the draft instead of the target",
      "bonus[b] = int(target_tok[b, v])", "bonus[b] = int(token[b, v])"),
+    ("accept", "the root counted as an accepted token",
+     "accept_len[b] = len(path) - 1", "accept_len[b] = len(path)"),
     ("accept", "a matching token anywhere in the tree accepted, not only among the children",
      "if int(parent[b, c]) == v and int(token[b, c]) == want]",
      "if c > v and int(token[b, c]) == want]"),
@@ -152,6 +182,10 @@ MUTANTS = [
      "v_new[dp, :, dr, :] = v_cache[sp, :, sr, :]", "v_new[dp, :, dr, :] = k_cache[sp, :, sr, :]"),
     ("compact_accepted_kv", "page and row of a position swapped",
      "return int(block_table[b, t // page]), t % page", "return int(block_table[b, t % page]), t // page"),
+    ("compact_accepted_kv", "source position without the context offset",
+     "sp, sr = where(b, c + int(accepted_nodes[b, i]))", "sp, sr = where(b, int(accepted_nodes[b, i]))"),
+    ("compact_accepted_kv", "destination one position late",
+     "dp, dr = where(b, c + i)", "dp, dr = where(b, c + i + 1)"),
 ]
 
 

@@ -547,6 +547,27 @@ def test_chain_when_k_is_one():
         assert s["token"][0, 1:n].tolist() == list(range(10, 10 + n - 1))
 
 
+@pytest.mark.parametrize("c", [2.0, 0.25])
+def test_utility_scales_with_the_cost_weights(c):
+    """Eq. 3 is homogeneous: multiplying lambda1 and lambda2 by c divides every
+    utility by c, so with tau divided by c the same tree is selected. For c a
+    power of two every IEEE operation scales exactly, so the scaled run is
+    bit-identical up to the factor; the root's utility is 1 / lambda1."""
+    rng = np.random.default_rng(21)
+    L, K = 5, 3
+    q = _random_qcond(rng, L, K)[None]
+    ids = np.stack([rng.permutation(30)[:K] for _ in range(L)]).astype(np.int32)[None]
+    root, ctx = np.array([2]), np.array([50])
+    a = O.select_subtree(q, ids, root, ctx, 1.0, 0.1, 0.05, 40)
+    b = O.select_subtree(q, ids, root, ctx, 1.0 * c, 0.1 * c, 0.05 / c, 40)
+    for k in ("n_nodes", "parent", "depth", "token", "slot", "pos_id", "reach"):
+        np.testing.assert_array_equal(a[k], b[k])
+    n = int(a["n_nodes"][0])
+    assert 1 < n < 40
+    np.testing.assert_array_equal(b["utility"][0, :n], (a["utility"][0, :n] / F32(c)).astype(F32))
+    assert b["utility"][0, 0] == F32(1.0 / c)
+
+
 def test_threshold_stops_selection():
     rng = np.random.default_rng(9)
     q = _random_qcond(rng, 4, 3)[None]
