@@ -79,6 +79,8 @@ MUTANTS = [
      "q[b, d, i] = e / e.sum()", "q[b, d, i] = e"),
     ("score_qcond", "marginal-product scores renormalised to the best sibling",
      "q[b, d, i] = np.exp(ell)", "q[b, d, i] = np.exp(ell - ell.max())"),
+    ("score_qcond", "marginal scorer's softmax taken over probabilities, not log-probabilities",
+     "ell[j] = float(logp[b, d, j])", "ell[j] = float(np.exp(logp[b, d, j]))"),
     # Eq. 2: reach
     ("reach_of_path", "q_cond indexed [child, parent]",
      "r *= float(q_cond_b[d, parent_slot, j])", "r *= float(q_cond_b[d, j, parent_slot])"),
@@ -97,6 +99,8 @@ MUTANTS = [
      "if n < 0 or n > L or any(j >= K for j in slots):", "if n < 0 or n >= L or any(j >= K for j in slots):"),
     ("path_reach", "the root treated as outside the trie",
      "if n < 0 or n > L or any(j >= K for j in slots):", "if n <= 0 or n > L or any(j >= K for j in slots):"),
+    ("path_reach", "edge depths counted from 1",
+     "for d, j in enumerate(slots):\n                r = F32(", "for d, j in enumerate(slots, 1):\n                r = F32("),
     # Eq. 3 and Algorithm 1
     ("utility_denominators", "cost term counted one level deeper",
      "F32(l1 + F32(l2 * F32(d)))", "F32(l1 + F32(l2 * F32(d + 1)))"),
@@ -146,6 +150,8 @@ MUTANTS = [
      "scale = 1.0 / D if scale is None else scale"),
     ("tree_verify_attn", "query heads mapped to KV heads interleaved",
      "kv = h // group", "kv = h % Hkv"),
+    ("tree_verify_attn", "query read with the KV head's index",
+     "s = scale * (Kb[visible, kv, :] @ q[b, i, h])", "s = scale * (Kb[visible, kv, :] @ q[b, i, kv])"),
     ("tree_verify_attn", "block table ignored (pages taken in logical order)",
      "pages = block_table[b, t // P]", "pages = t // P"),
     ("tree_verify_attn", "tree mask read transposed",
