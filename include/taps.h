@@ -97,6 +97,10 @@ int taps_version(void);
  * Limits: 1 <= K <= min(32, V), 1 <= V <= 262143. Logits may be -inf
  * (probability 0, no entropy contribution) but not +inf or NaN, and every row
  * needs at least K finite logits for the top-K to be meaningful.
+ * Device-side waits: the kernel that serves a few rows waits for the bulk
+ * copies of its logits slice with a bound of about 2 s and then carries on
+ * either way. There is no status word to report an expired wait: it would
+ * need a copy from the caller's memory that never completes.
  * ---------------------------------------------------------------------- */
 size_t taps_topk_marginals_workspace_bytes(int B, int L, int V, int K);
 int taps_topk_marginals(const void* logits, int dtype, int64_t row_stride,
