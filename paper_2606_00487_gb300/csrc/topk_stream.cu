@@ -18,9 +18,11 @@
 // maximum of the first stage (at least KP elements reach it). When the list
 // grows past 128 entries it is compacted (ranked by counting): its KP-th
 // largest key becomes the threshold and only the KP keys above it stay
-// listed, so that the threshold soon follows the row's running top-KP. A stage that overflows
-// the list (1,024 entries) is listed again above the raised threshold, from
-// the copy still in shared memory. At the end the list is ranked by counting.
+// listed, so that the threshold soon follows the row's running top-KP. A
+// stage that overflows the list (1,024 entries) is listed again above the
+// raised threshold, from the copy still in shared memory; each compaction
+// raises the threshold strictly (the listed keys are distinct), so the
+// re-listing ends. At the end the list is ranked by counting.
 #include <algorithm>
 #include <atomic>
 
