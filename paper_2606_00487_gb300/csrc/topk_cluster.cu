@@ -17,9 +17,10 @@
 //     shared memory and ranked by counting.
 // Every CTA then writes its top-KP and statistics into the shared memory of the
 // cluster's first CTA (distributed shared memory); after one cluster barrier
-// one warp of that CTA merges them by rank and writes the row's outputs. No partial record
-// goes through global memory, no counter, no workspace. The host launches this
-// kernel only when every row's cluster can be resident at once; otherwise
+// one warp of that CTA merges them by rank and writes the row's outputs. No
+// partial record goes through global memory, no counter, no workspace. The
+// host launches this kernel only when every row's cluster can be resident at
+// once; otherwise topk_stream_kernel (topk_stream.cu, from 304 rows) or
 // topk_marginals_kernel (topk.cu) runs.
 #include <algorithm>
 #include <mutex>
