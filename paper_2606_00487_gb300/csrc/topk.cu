@@ -12,6 +12,12 @@
 // rank into one partial record. The last CTA of a row (an atomic ticket,
 // reset after use) merges the partials by rank and writes the row's outputs.
 // No CTA waits on another.
+//
+// taps_topk_marginals first offers the rows to two specialised kernels: one
+// thread-block cluster per row when every row's cluster fits on the GPU at
+// once (topk_cluster.cu, batch-1 rounds), one CTA per row from 304 rows
+// (topk_stream.cu, batched rounds); this kernel serves the shapes in between
+// (e.g. 128 rows) and unaligned logits.
 #include <algorithm>
 #include <atomic>
 #include <mutex>
